@@ -1,0 +1,295 @@
+"""Plain, slow, fp64 CPU oracle for COVER's override-attention and seed-scoring path.
+
+TEST INFRASTRUCTURE ONLY. Nothing in the product path may import this module:
+only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline /
+reference leg use it. It shares no code with the CUDA kernels or their host
+glue; it works on numpy float64 arrays that the caller widened exactly from the
+stored (fp32 or bf16) inputs.
+
+Everything here is written from the paper's definitions:
+
+* §5.1 "Dual-View Feed Forward through KV Cache Override": the overridden memory
+  K', V' (seed columns hold the cached states), attention of every query over
+  K', V' with softmax scale 1/sqrt(d), and, for a seed query i, the
+  leave-one-out key/value set whose diagonal entry is restored to the pair
+  (k_i, v_i) computed from the masked input.
+* Appendix B (B.1 notation, Lemma B.1, B.3 weights, B.4 outputs): the closed
+  form diagonal correction alpha_i, delta_i, r_i and the corrected output.
+* §3 (drafting): greedy token argmax p and confidence max p.
+* §6.1: entropy-ordered greedy unmasking (Shannon entropy of p).
+* §5.3: uncertainty u(j) = -log p_j(y_j), Score(j) = u (1 + d_in)/(1 + d_out),
+  top-k seed selection over eligible positions.
+
+Readings of points the paper leaves open (numbered as in the design notes):
+the cached inputs already hold the overridden memory K', V' (R1); the masked
+pairs (k_i, v_i) come as a compact [B, Hkv, S, D] buffer whose row s belongs to
+position seed_idx[b, s] (R2); grouped-query heads map hkv = hq // (Hq/Hkv)
+(R3); no causal mask (R4); scale 1/sqrt(D) (R5); the lse of a seed row is that
+of its corrected distribution (R6); out-of-range seeds are ignored and, among
+duplicates, the lowest slot wins (R7); ties in argmax / top-k go to the lower
+index (R9); entropy is natural-log Shannon entropy at temperature 1 (R10);
+without current tokens y = argmax (R11); absent d_in / d_out are 0 (R12);
+top-k takes the largest scores (R13).
+
+Every function is pinned by ``tests/test_oracle_pins.py`` against closed forms,
+hand-worked fixtures, a library routine (torch float64 SDPA) and brute force.
+"""
+from __future__ import annotations
+
+import math
+from typing import Optional, Sequence
+
+import numpy as np
+
+TILE_ROWS = 128  # row-tile height of the seed bitmap (a build structure, not the paper's)
+
+
+# ----------------------------------------------------------------------------
+# Seed routing (seed set semantics, §3 "Decoding protocol" and §5.1)
+# ----------------------------------------------------------------------------
+
+def route_seeds(seed_idx: np.ndarray, L: int):
+    """Map each position of each batch row to the slot of the seed that names it.
+
+    seed_idx: int [B, S]. Returns (slot [B, L] int32 with -1 for non-seeds,
+    bitmap [B, ceil(L/128), 4] uint32 with bit (r % 32) of word (r % 128) // 32
+    of tile r // 128 set iff slot[r] >= 0, n_invalid = number of entries that
+    are out of [0, L) or repeat an earlier slot's position).
+    """
+    seed_idx = np.asarray(seed_idx)
+    B = seed_idx.shape[0]
+    S = seed_idx.shape[1] if seed_idx.ndim == 2 else 0
+    slot = np.full((B, L), -1, dtype=np.int32)
+    n_invalid = 0
+    for b in range(B):
+        for s in range(S):
+            p = int(seed_idx[b, s])
+            if p < 0 or p >= L:
+                n_invalid += 1
+                continue
+            if slot[b, p] >= 0:
+                n_invalid += 1          # duplicate: the earlier (lower) slot keeps the position
+                continue
+            slot[b, p] = s
+    n_tiles = (L + TILE_ROWS - 1) // TILE_ROWS
+    bitmap = np.zeros((B, n_tiles, 4), dtype=np.uint32)
+    for b in range(B):
+        for r in range(L):
+            if slot[b, r] >= 0:
+                t, w, bit = r // TILE_ROWS, (r % TILE_ROWS) // 32, r % 32
+                bitmap[b, t, w] |= np.uint32(1) << np.uint32(bit)
+    return slot, bitmap, n_invalid
+
+
+# ----------------------------------------------------------------------------
+# Attention: the explicit two-view definition (§5.1, Appendix B.1)
+# ----------------------------------------------------------------------------
+
+def _softmax_row(z: np.ndarray):
+    """Naive softmax with max subtraction; returns (weights, natural-log lse)."""
+    m = np.max(z)
+    e = np.exp(z - m)
+    Z = np.sum(e)
+    return e / Z, m + math.log(Z)
+
+
+def view_for_row(kc_h: np.ndarray, vc_h: np.ndarray, i: int, masked_pair=None):
+    """Key/value set seen by query i (§5.1, Appendix B.1).
+
+    kc_h, vc_h: [L, D] overridden memory K', V' of one KV head. For a seed query
+    the diagonal entry is restored to the masked-input pair (k_i, v_i); every
+    other entry stays K', V'. Non-seed queries see K', V' unchanged.
+    """
+    if masked_pair is None:
+        return kc_h, vc_h
+    K = kc_h.copy()
+    V = vc_h.copy()
+    K[i] = masked_pair[0]
+    V[i] = masked_pair[1]
+    return K, V
+
+
+def attention_row(q_i: np.ndarray, K: np.ndarray, V: np.ndarray):
+    """o_i = softmax(K q_i / sqrt(d)) V and its lse, for one query over one key/value set."""
+    d = q_i.shape[-1]
+    z = (K @ q_i) / math.sqrt(d)
+    w, lse = _softmax_row(z)
+    return w @ V, lse, w
+
+
+def override_attention_rows(q, kc, vc, km, vm, seed_idx, b: int, hq: int, rows: Sequence[int]):
+    """Outputs of the listed query rows of head (b, hq), each from its own explicit view."""
+    B, Hq, L, D = q.shape
+    Hkv = kc.shape[1]
+    hkv = hq // (Hq // Hkv)
+    slot, _, _ = route_seeds(seed_idx[b:b + 1], L) if seed_idx is not None and seed_idx.size else (
+        np.full((1, L), -1, np.int32), None, 0)
+    out = np.zeros((len(rows), D))
+    lse = np.zeros(len(rows))
+    for n, i in enumerate(rows):
+        s = int(slot[0, i])
+        pair = (km[b, hkv, s], vm[b, hkv, s]) if s >= 0 else None
+        K, V = view_for_row(kc[b, hkv], vc[b, hkv], i, pair)
+        out[n], lse[n], _ = attention_row(q[b, hq, i], K, V)
+    return out, lse
+
+
+def override_attention(q, kc, vc, km, vm, seed_idx):
+    """Full two-view attention output and lse for every (b, hq, i).
+
+    q [B,Hq,L,D], kc/vc [B,Hkv,L,D] (= K', V'), km/vm [B,Hkv,S,D],
+    seed_idx [B,S]. Non-seed rows are plain attention over K', V' (computed a
+    head at a time with a matmul); seed rows go through their explicit
+    leave-one-out view one by one.
+    """
+    B, Hq, L, D = q.shape
+    Hkv = kc.shape[1]
+    G = Hq // Hkv
+    S = 0 if seed_idx is None else seed_idx.shape[1]
+    slot = route_seeds(seed_idx, L)[0] if S else np.full((B, L), -1, np.int32)
+    out = np.zeros((B, Hq, L, D))
+    lse = np.zeros((B, Hq, L))
+    for b in range(B):
+        for hq in range(Hq):
+            hkv = hq // G
+            Kp, Vp = kc[b, hkv], vc[b, hkv]
+            z = (q[b, hq] @ Kp.T) / math.sqrt(D)          # [L, L]
+            m = z.max(axis=1, keepdims=True)
+            e = np.exp(z - m)
+            Z = e.sum(axis=1, keepdims=True)
+            out[b, hq] = (e / Z) @ Vp
+            lse[b, hq] = (m + np.log(Z))[:, 0]
+            for i in np.nonzero(slot[b] >= 0)[0]:
+                s = int(slot[b, i])
+                K, V = view_for_row(Kp, Vp, int(i), (km[b, hkv, s], vm[b, hkv, s]))
+                out[b, hq, i], lse[b, hq, i], _ = attention_row(q[b, hq, i], K, V)
+    return out, lse
+
+
+def override_attention_closed_form(q, kc, vc, km, vm, seed_idx):
+    """The same result through Appendix B's closed form (Lemma B.1, B.3, B.4).
+
+    One attention pass over K', V' for all rows, then for each seed row:
+    alpha_i = w_ovr[i, i], delta_i = q_i (k_i - k'_i) / sqrt(d),
+    r_i = 1 + alpha_i (exp(delta_i) - 1),
+    o_i = (o_ovr_i - alpha_i v'_i + alpha_i exp(delta_i) v_i) / r_i,
+    lse_i = lse_ovr_i + ln r_i (the normaliser changes by the factor r_i).
+    """
+    B, Hq, L, D = q.shape
+    Hkv = kc.shape[1]
+    G = Hq // Hkv
+    S = 0 if seed_idx is None else seed_idx.shape[1]
+    slot = route_seeds(seed_idx, L)[0] if S else np.full((B, L), -1, np.int32)
+    out = np.zeros((B, Hq, L, D))
+    lse = np.zeros((B, Hq, L))
+    for b in range(B):
+        for hq in range(Hq):
+            hkv = hq // G
+            Kp, Vp = kc[b, hkv], vc[b, hkv]
+            s_ovr = (q[b, hq] @ Kp.T) / math.sqrt(D)
+            m = s_ovr.max(axis=1, keepdims=True)
+            e = np.exp(s_ovr - m)
+            Z = e.sum(axis=1, keepdims=True)
+            w_ovr = e / Z
+            o_ovr = w_ovr @ Vp
+            lse_ovr = (m + np.log(Z))[:, 0]
+            out[b, hq] = o_ovr
+            lse[b, hq] = lse_ovr
+            for i in np.nonzero(slot[b] >= 0)[0]:
+                s = int(slot[b, i])
+                k_i, v_i = km[b, hkv, s], vm[b, hkv, s]
+                alpha = w_ovr[i, i]
+                delta = float(q[b, hq, i] @ (k_i - Kp[i])) / math.sqrt(D)
+                r = 1.0 + alpha * (math.exp(delta) - 1.0)
+                out[b, hq, i] = (o_ovr[i] - alpha * Vp[i] + alpha * math.exp(delta) * v_i) / r
+                lse[b, hq, i] = lse_ovr[i] + math.log(r)
+    return out, lse
+
+
+def corrected_weights_row(q, kc, vc, km, vm, seed_idx, b: int, hq: int, i: int):
+    """Attention weights of row i under its own view (Appendix B.3), for sum-to-one checks."""
+    B, Hq, L, D = q.shape
+    hkv = hq // (Hq // kc.shape[1])
+    slot = route_seeds(seed_idx[b:b + 1], L)[0][0] if seed_idx is not None and seed_idx.size else (
+        np.full(L, -1, np.int32))
+    s = int(slot[i])
+    pair = (km[b, hkv, s], vm[b, hkv, s]) if s >= 0 else None
+    K, V = view_for_row(kc[b, hkv], vc[b, hkv], i, pair)
+    return attention_row(q[b, hq, i], K, V)[2]
+
+
+# ----------------------------------------------------------------------------
+# Per-position scoring (§3 drafting, §6.1 entropy, §5.3 seed score)
+# ----------------------------------------------------------------------------
+
+def score_rows(logits: np.ndarray, cur_tok=None, d_in=None, d_out=None):
+    """Per-row confidence, entropy, greedy token, uncertainty and seed score.
+
+    logits: float64 [N, V] (exact widening of the bf16 values). For each row,
+    p = softmax(x) at temperature 1; c = max_v p(v) (§3); y_hat = the first
+    index attaining the maximum logit (§3, ties to the lower index); H =
+    -sum_v p(v) ln p(v) (§6.1); u = -ln p(y) with y = cur_tok, or y_hat when no
+    current tokens are given (§5.3); Score = u (1 + d_in) / (1 + d_out) with
+    absent d_in / d_out taken as 0 (§5.3).
+    Returns dict of float64 / int64 arrays: maxprob, entropy, argmax, u, score.
+    """
+    x = np.asarray(logits, dtype=np.float64)
+    N, V = x.shape
+    maxprob = np.zeros(N)
+    entropy = np.zeros(N)
+    argmax = np.zeros(N, dtype=np.int64)
+    u = np.zeros(N)
+    score = np.zeros(N)
+    for n in range(N):
+        row = x[n]
+        m = row.max()
+        y_hat = int(np.argmax(row))            # first occurrence of the maximum
+        e = np.exp(row - m)
+        Z = e.sum()
+        p = e / Z
+        logp = (row - m) - math.log(Z)
+        maxprob[n] = p.max()
+        entropy[n] = -np.sum(p * logp)
+        argmax[n] = y_hat
+        y = y_hat if cur_tok is None else int(cur_tok[n])
+        u[n] = -logp[y]
+        din = 0.0 if d_in is None else float(d_in[n])
+        dout = 0.0 if d_out is None else float(d_out[n])
+        score[n] = u[n] * (1.0 + din) / (1.0 + dout)
+    return dict(maxprob=maxprob, entropy=entropy, argmax=argmax, u=u, score=score)
+
+
+def topk_select(score: np.ndarray, n_seq: int, k: int, eligible=None):
+    """Top-k seed selection per sequence segment (§5.3).
+
+    The N rows split into n_seq equal consecutive segments. Within a segment the
+    eligible rows are ordered by score, largest first, ties to the lower index;
+    the first k are taken. Returned indices are offsets within the segment;
+    missing entries (fewer than k eligible rows) are -1 with score -inf.
+    """
+    score = np.asarray(score)
+    N = score.shape[0]
+    per = N // n_seq
+    idx = np.full((n_seq, k), -1, dtype=np.int64)
+    val = np.full((n_seq, k), -np.inf)
+    for g in range(n_seq):
+        cand = [j for j in range(per) if eligible is None or eligible[g * per + j]]
+        ranked = sorted(cand, key=lambda j: (-float(score[g * per + j]), j))
+        for t, j in enumerate(ranked[:k]):
+            idx[g, t] = j
+            val[g, t] = score[g * per + j]
+    return idx, val
+
+
+def topk_margin(score: np.ndarray, n_seq: int, k: int, eligible=None):
+    """Per segment, the gap between the k-th and (k+1)-th largest eligible score (inf if none)."""
+    score = np.asarray(score, dtype=np.float64)
+    N = score.shape[0]
+    per = N // n_seq
+    gaps = np.full(n_seq, np.inf)
+    for g in range(n_seq):
+        vals = [score[g * per + j] for j in range(per) if eligible is None or eligible[g * per + j]]
+        vals.sort(reverse=True)
+        if len(vals) > k:
+            gaps[g] = vals[k - 1] - vals[k]
+    return gaps
