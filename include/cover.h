@@ -1,0 +1,156 @@
+/*
+ * cover.h - C ABI of the COVER override-attention and seed-scoring kernels
+ * (single GB300 GPU, sm_103a).
+ *
+ * COVER ("Stop the Flip-Flop: Context-Preserving Verification for Fast
+ * Revocable Diffusion Decoding") verifies previously decoded "seed" positions
+ * in the same forward pass that drafts new tokens. Section 5.1: the seeds are
+ * masked in the input, their key/value columns are overridden with the states
+ * cached at the previous step (memory K', V'), every query attends once over
+ * K', V', and each seed query's own diagonal entry is restored to the pair
+ * (k_i, v_i) computed from the masked input (leave-one-out view). Appendix B
+ * gives the closed form of that diagonal correction.
+ *
+ * Conventions for every entry point:
+ *  - Pointers are DEVICE pointers owned by the caller, unless stated otherwise.
+ *    The library allocates no device memory and keeps no per-call state.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream). Argument errors are returned synchronously, before any launch.
+ *  - Kernels never trap. A kernel that gives up on an internal wait (bounded at
+ *    about one second) records COVER_ERR_DEVICE_TIMEOUT in a per-device status
+ *    word; read and clear it with cover_device_status().
+ *  - Tensors are dense and contiguous (row-major, last index fastest).
+ */
+#ifndef COVER_H_
+#define COVER_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  COVER_OK = 0,
+  COVER_ERR_INVALID_ARG = -1,    /* null required pointer, bad size, misaligned pointer */
+  COVER_ERR_UNSUPPORTED = -2,    /* valid request outside what the kernels implement (e.g. head dim) */
+  COVER_ERR_CUDA = -3,           /* a CUDA runtime call or launch failed */
+  COVER_ERR_DEVICE_TIMEOUT = -4  /* a kernel gave up on a bounded internal wait (status word only) */
+} cover_status_t;
+
+/*
+ * Two-view override attention, bf16 in / bf16 out, fp32 accumulation.
+ * Section 5.1 (Attn(Q, K', V') over the overridden memory, softmax scale
+ * 1/sqrt(d)) and Appendix B.1-B.4 (diagonal correction of seed queries).
+ *
+ *   q          [B, Hq,  L, D] bf16  queries from the masked-seed input
+ *   k_cached   [B, Hkv, L, D] bf16  overridden memory K' (seed columns already
+ *   v_cached   [B, Hkv, L, D] bf16  hold the previous step's cached states)
+ *   k_seedmask [B, Hkv, n_seeds, D] bf16  row s = key   of position seed_idx[b, s]
+ *   v_seedmask [B, Hkv, n_seeds, D] bf16  row s = value of position seed_idx[b, s]
+ *                                   computed from the masked input (may be NULL
+ *                                   when n_seeds == 0)
+ *   seed_idx   [B, n_seeds] int32   seed positions per batch row, any order.
+ *                                   Entries outside [0, L) are ignored; if a
+ *                                   position repeats, the lowest slot s is used.
+ *   out        [B, Hq, L, D] bf16   o_i (corrected for seed rows)
+ *   lse        [B, Hq, L] fp32      natural-log log-sum-exp of the scaled
+ *                                   scores of each row's own view (NULL = skip)
+ *
+ * Query head hq reads KV head hq / (Hq / Hkv) (contiguous groups). No causal
+ * mask. For non-seed rows the result is plain attention over K', V'; for a
+ * seed row i the diagonal term uses (k_i, v_i) instead of (k'_i, v'_i).
+ *
+ * Requirements: D == 128 (else COVER_ERR_UNSUPPORTED); B, Hq, Hkv, L >= 1;
+ * Hq % Hkv == 0; 0 <= n_seeds <= L; q, k_cached, v_cached, out, k_seedmask,
+ * v_seedmask 16-byte aligned; lse 4-byte aligned. Any L >= 1 is supported.
+ * Otherwise COVER_ERR_INVALID_ARG. The inputs must not alias out / lse.
+ */
+int cover_attn_fwd(const void* q, const void* k_cached, const void* v_cached,
+                   const void* k_seedmask, const void* v_seedmask,
+                   const int32_t* seed_idx, int n_seeds,
+                   int B, int Hq, int Hkv, int L, int D,
+                   void* out, float* lse, void* stream);
+
+/*
+ * The same operation in fp32 throughout (float tensors, fp32 FMA on CUDA
+ * cores, accurate expf). Intended for small fp32 checks. D in {64, 128}.
+ * Same layouts, ownership and errors as cover_attn_fwd (4-byte alignment).
+ */
+int cover_attn_fwd_f32(const float* q, const float* k_cached, const float* v_cached,
+                       const float* k_seedmask, const float* v_seedmask,
+                       const int32_t* seed_idx, int n_seeds,
+                       int B, int Hq, int Hkv, int L, int D,
+                       float* out, float* lse, void* stream);
+
+/*
+ * Seed routing as the attention kernels see it (seed-set semantics of
+ * Sections 3 and 5.1), exported for checking.
+ *   slot_out   [B, L] int32: slot s of the seed naming position r, else -1
+ *   bitmap_out [B, ceil(L/128), 4] uint32: bit r%32 of word (r%128)/32 of
+ *              tile r/128 is set iff slot_out[b, r] >= 0
+ *   n_invalid_out [1] int32: entries out of [0, L) plus repeated positions
+ * seed_idx may be NULL when n_seeds == 0. Requirements: B, L >= 1,
+ * 0 <= n_seeds <= L (else COVER_ERR_INVALID_ARG).
+ */
+int cover_seed_route(const int32_t* seed_idx, int n_seeds, int B, int L,
+                     int32_t* slot_out, uint32_t* bitmap_out, int32_t* n_invalid_out,
+                     void* stream);
+
+/*
+ * Bytes of device workspace cover_score_fwd needs for n_seq segments.
+ * The caller allocates it once, fills it with zeros, and may pass the same
+ * buffer to every later call (each call leaves it zeroed again). Calls that
+ * share one workspace must not run concurrently on the GPU.
+ */
+size_t cover_score_workspace_bytes(int n_seq);
+
+/*
+ * Fused per-position scoring over the vocabulary and top-k seed selection.
+ * Section 3 (greedy token y_hat = argmax p, confidence c = max p), Section 6.1
+ * (entropy-ordered unmasking: H = -sum p ln p), Section 5.3 (uncertainty
+ * u = -log p(y), Score = u (1 + d_in)/(1 + d_out), top-k over eligible rows).
+ *
+ *   logits  [N, V] bf16   one row per scored position, softmax at temperature 1
+ *   n_seq               rows split into n_seq equal consecutive segments
+ *                       (sequences); top-k is taken per segment
+ *   cur_tok [N] int32   current token y of each row; NULL => y = argmax row
+ *   d_in, d_out [N] f32 influence / drift terms of the score; NULL => 0
+ *   eligible [N] uint8  nonzero = row may be selected; NULL => all rows
+ *   topk                k per segment (0 <= k <= N / n_seq)
+ * Outputs (per row): maxprob = c, entropy = H, argmax = y_hat (lowest index
+ * among equal maxima), score = Score. Per segment: topk_idx [n_seq, topk]
+ * (row offsets within the segment, by score descending then index
+ * ascending; -1 where fewer than k rows are eligible) and topk_score
+ * [n_seq, topk] (NULL = skip; -inf where idx is -1).
+ * workspace: cover_score_workspace_bytes(n_seq) zero-filled bytes (see above).
+ *
+ * Requirements: N, V >= 1; 1 <= n_seq; N % n_seq == 0; N / n_seq <= 4096;
+ * logits 16-byte aligned (any V; rows need not be 16-byte aligned).
+ * A cur_tok entry outside [0, V) yields NaN u and score for that row.
+ * Non-finite logits give unspecified results. Otherwise COVER_ERR_INVALID_ARG.
+ */
+int cover_score_fwd(const void* logits, int N, int V, int n_seq,
+                    const int32_t* cur_tok, const float* d_in, const float* d_out,
+                    const uint8_t* eligible, int topk,
+                    float* maxprob, float* entropy, int32_t* argmax, float* score,
+                    int32_t* topk_idx, float* topk_score,
+                    void* workspace, void* stream);
+
+/*
+ * Synchronises `stream`, then returns and clears the current device's status
+ * word: COVER_OK, or COVER_ERR_DEVICE_TIMEOUT if a kernel gave up on a
+ * bounded wait since the last call. Returns COVER_ERR_CUDA if the
+ * synchronisation itself fails.
+ */
+int cover_device_status(void* stream);
+
+/* Static, human-readable name of a status code. Never NULL. */
+const char* cover_status_str(int code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* COVER_H_ */

@@ -1,0 +1,178 @@
+"""Python binding of the COVER kernel library: same names as the C ABI.
+
+Each function checks tensor dtypes / devices / contiguity, reads the sizes off
+the tensors, and calls the C entry point on the current CUDA stream. All
+arithmetic runs in the CUDA kernels; torch only provides device memory and
+streams.
+"""
+from __future__ import annotations
+
+from typing import Optional
+
+import torch
+
+from . import _lib
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _need(t: torch.Tensor, name: str, dtype, ndim: int):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims, got {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def _attn(fn_name, dtype, q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, out, lse, want_lse, stream):
+    _need(q, "q", dtype, 4)
+    _need(k_cached, "k_cached", dtype, 4)
+    _need(v_cached, "v_cached", dtype, 4)
+    B, Hq, L, D = q.shape
+    Hkv = k_cached.shape[1]
+    if tuple(k_cached.shape) != (B, Hkv, L, D) or tuple(v_cached.shape) != (B, Hkv, L, D):
+        raise ValueError("k_cached / v_cached must be [B, Hkv, L, D] matching q")
+    n_seeds = 0 if seed_idx is None else int(seed_idx.shape[1])
+    if n_seeds > 0:
+        _need(seed_idx, "seed_idx", torch.int32, 2)
+        _need(k_seedmask, "k_seedmask", dtype, 4)
+        _need(v_seedmask, "v_seedmask", dtype, 4)
+        if tuple(seed_idx.shape) != (B, n_seeds):
+            raise ValueError("seed_idx must be [B, S]")
+        if tuple(k_seedmask.shape) != (B, Hkv, n_seeds, D) or tuple(v_seedmask.shape) != (B, Hkv, n_seeds, D):
+            raise ValueError("k_seedmask / v_seedmask must be [B, Hkv, S, D]")
+    if out is None:
+        out = torch.empty_like(q)
+    else:
+        _need(out, "out", dtype, 4)
+    if lse is None and want_lse:
+        lse = torch.empty((B, Hq, L), dtype=torch.float32, device=q.device)
+    elif lse is not None:
+        _need(lse, "lse", torch.float32, 3)
+    lib = _lib.load()
+    code = getattr(lib, fn_name)(
+        _ptr(q), _ptr(k_cached), _ptr(v_cached),
+        _ptr(k_seedmask) if n_seeds else None, _ptr(v_seedmask) if n_seeds else None,
+        _ptr(seed_idx) if n_seeds else None, n_seeds, B, Hq, Hkv, L, D,
+        _ptr(out), _ptr(lse), _stream(stream))
+    _lib.check(fn_name, code)
+    return out, lse
+
+
+def cover_attn_fwd(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, seed_idx=None, *,
+                   out=None, lse=None, want_lse=True, stream=None):
+    """Two-view override attention (bf16). Returns (out [B,Hq,L,D] bf16, lse [B,Hq,L] f32 or None)."""
+    return _attn("cover_attn_fwd", torch.bfloat16, q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx,
+                 out, lse, want_lse, stream)
+
+
+def cover_attn_fwd_f32(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, seed_idx=None, *,
+                       out=None, lse=None, want_lse=True, stream=None):
+    """Two-view override attention in fp32 (CUDA cores)."""
+    return _attn("cover_attn_fwd_f32", torch.float32, q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx,
+                 out, lse, want_lse, stream)
+
+
+def cover_seed_route(seed_idx: Optional[torch.Tensor], B: int, L: int, *, device=None, stream=None):
+    """Seed routing as the kernels see it: (slot [B,L] int32, bitmap [B,ceil(L/128),4] int32 bits, n_invalid)."""
+    n_seeds = 0 if seed_idx is None else int(seed_idx.shape[1])
+    if n_seeds:
+        _need(seed_idx, "seed_idx", torch.int32, 2)
+        device = seed_idx.device
+    device = device or torch.device("cuda")
+    slot = torch.empty((B, L), dtype=torch.int32, device=device)
+    bitmap = torch.empty((B, (L + 127) // 128, 4), dtype=torch.int32, device=device)
+    n_invalid = torch.empty((1,), dtype=torch.int32, device=device)
+    code = _lib.load().cover_seed_route(_ptr(seed_idx) if n_seeds else None, n_seeds, B, L, _ptr(slot),
+                                        _ptr(bitmap), _ptr(n_invalid), _stream(stream))
+    _lib.check("cover_seed_route", code)
+    return slot, bitmap, n_invalid
+
+
+def cover_score_workspace_bytes(n_seq: int) -> int:
+    return int(_lib.load().cover_score_workspace_bytes(int(n_seq)))
+
+
+def score_workspace(n_seq: int, device=None) -> torch.Tensor:
+    """A zero-filled workspace for cover_score_fwd (reusable across calls on one stream)."""
+    nbytes = cover_score_workspace_bytes(n_seq)
+    return torch.zeros((max(nbytes, 4) + 3) // 4, dtype=torch.int32, device=device or "cuda")
+
+
+def cover_score_fwd(logits, n_seq: int, topk: int, *, cur_tok=None, d_in=None, d_out=None, eligible=None,
+                    workspace=None, out=None, stream=None):
+    """Fused vocabulary scoring + per-segment top-k.
+
+    Returns a dict of CUDA tensors: maxprob, entropy, argmax, score [N];
+    topk_idx [n_seq, topk] int32 and topk_score [n_seq, topk] f32.
+    """
+    _need(logits, "logits", torch.bfloat16, 2)
+    N, V = logits.shape
+    dev = logits.device
+    if cur_tok is not None:
+        _need(cur_tok, "cur_tok", torch.int32, 1)
+    if d_in is not None:
+        _need(d_in, "d_in", torch.float32, 1)
+    if d_out is not None:
+        _need(d_out, "d_out", torch.float32, 1)
+    if eligible is not None:
+        _need(eligible, "eligible", torch.uint8, 1)
+    if out is None:
+        out = dict(
+            maxprob=torch.empty(N, dtype=torch.float32, device=dev),
+            entropy=torch.empty(N, dtype=torch.float32, device=dev),
+            argmax=torch.empty(N, dtype=torch.int32, device=dev),
+            score=torch.empty(N, dtype=torch.float32, device=dev),
+            topk_idx=torch.empty((n_seq, max(topk, 0)), dtype=torch.int32, device=dev),
+            topk_score=torch.empty((n_seq, max(topk, 0)), dtype=torch.float32, device=dev),
+        )
+    if workspace is None and topk > 0:
+        workspace = score_workspace(n_seq, dev)
+    code = _lib.load().cover_score_fwd(
+        _ptr(logits), N, V, n_seq, _ptr(cur_tok), _ptr(d_in), _ptr(d_out), _ptr(eligible), topk,
+        _ptr(out["maxprob"]), _ptr(out["entropy"]), _ptr(out["argmax"]), _ptr(out["score"]),
+        _ptr(out["topk_idx"]) if topk > 0 else None, _ptr(out["topk_score"]) if topk > 0 else None,
+        _ptr(workspace), _stream(stream))
+    _lib.check("cover_score_fwd", code)
+    return out
+
+
+def cover_device_status(stream=None) -> int:
+    """Synchronise the stream; return and clear the device status word (0 = OK)."""
+    return int(_lib.load().cover_device_status(_stream(stream)))
+
+
+def cover_status_str(code: int) -> str:
+    return _lib.status_str(code)
+
+
+def cover_debug_umma_tile(a, b, p, v, *, stream=None):
+    for name, t in (("a", a), ("b", b), ("p", p), ("v", v)):
+        _need(t, name, torch.bfloat16, 2)
+        if tuple(t.shape) != (128, 128):
+            raise ValueError(f"{name} must be [128, 128]")
+    c1 = torch.empty((128, 128), dtype=torch.float32, device=a.device)
+    c2 = torch.empty((128, 128), dtype=torch.float32, device=a.device)
+    code = _lib.load().cover_debug_umma_tile(_ptr(a), _ptr(b), _ptr(p), _ptr(v), _ptr(c1), _ptr(c2),
+                                             _stream(stream))
+    _lib.check("cover_debug_umma_tile", code)
+    return c1, c2
+
+
+def cover_debug_wait_timeout(limit_us: int, *, stream=None) -> None:
+    _lib.check("cover_debug_wait_timeout", _lib.load().cover_debug_wait_timeout(int(limit_us), _stream(stream)))

@@ -1,0 +1,409 @@
+// attn_bf16_sm103.cu - two-view override attention, bf16, tcgen05 tensor cores.
+//
+// What it computes (Section 5.1, Appendix B): for every query row i of head
+// (b, hq), attention over the overridden memory K', V' of KV head
+// hq / (Hq / Hkv), scale 1/sqrt(d), no causal mask; for a seed row the
+// diagonal entry uses the masked-input pair (k_i, v_i) instead of (k'_i, v'_i)
+// (leave-one-out view). The diagonal correction of Appendix B is applied in
+// exclusion form: the cached diagonal score of a seed row is set to -inf
+// inside the online softmax (only in the one KV tile that holds the diagonal),
+// and the masked self term e^{s_self - m} v_i is merged into (m, l, O) in the
+// epilogue. Equal to the closed form in exact arithmetic; it never divides by
+// r_i, and a seed row never reads k'_i, v'_i while a non-seed row never reads
+// the masked buffer.
+//
+// Structure (one CTA per 256 query rows of one head, 1 CTA per SM):
+//   warps 0-3  softmax + epilogue of Q tile 0 (thread = row)
+//   warps 4-7  softmax + epilogue of Q tile 1
+//   warp  8    tensor-memory allocation; lane 0 issues tcgen05.mma
+//   warp  9    lane 0 issues TMA loads (Q once, K/V through a 2-stage ring)
+// Tensor memory (512 columns): S0 | S1 | O0 | O1, 128 fp32 columns each; the
+// bf16 probabilities P of tile t overwrite the first 64 columns of S_t and
+// feed the P.V product straight from tensor memory.
+// Per KV tile j the MMA issue order is PV(0, j-1), S(0, j), PV(1, j-1), S(1, j)
+// so that one Q tile's softmax overlaps the other tile's products.
+// The running max is updated lazily: O is rescaled only when a row's max grows
+// by more than 2^8.
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "kernels.cuh"
+#include "ptx.cuh"
+#include "route.cuh"
+#include "tmap.cuh"
+
+namespace cover {
+namespace {
+
+constexpr int kD = 128;
+constexpr int kBM = 128;                  // rows per Q tile
+constexpr int kBN = 128;                  // keys per KV tile
+constexpr int kNQ = 2;                    // Q tiles per CTA
+constexpr int kRowsPerCta = kNQ * kBM;
+constexpr int kStages = 2;
+constexpr int kTileBytes = kBM * kD * 2;  // 32 KB
+constexpr int kBoxBytes = kTileBytes / 2; // one 64-column, 128-byte-swizzled box
+constexpr int kThreads = 320;
+constexpr int kMmaWarp = 8;
+constexpr int kTmaWarp = 9;
+constexpr float kRescaleThreshold = 8.0f;  // log2 units
+
+struct AttnSmem {
+  uint8_t q[kNQ][kTileBytes];
+  uint8_t k[kStages][kTileBytes];
+  uint8_t v[kStages][kTileBytes];
+  uint64_t bar_q;
+  uint64_t bar_k_full[kStages];
+  uint64_t bar_k_empty[kStages];
+  uint64_t bar_v_full[kStages];
+  uint64_t bar_v_empty[kStages];
+  uint64_t bar_s_full[kNQ];
+  uint64_t bar_p_full[kNQ];
+  uint64_t bar_o_full[kNQ];
+  uint64_t bar_drain;
+  uint32_t tmem_base;
+  int abort;
+  int slot[kRowsPerCta];
+};
+
+__device__ __forceinline__ uint32_t col_s(int qt) { return qt * 128u; }
+__device__ __forceinline__ uint32_t col_o(int qt) { return 256u + qt * 128u; }
+
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  const bool ok = mbar_wait(bar, parity, abort);
+  return __all_sync(0xffffffffu, ok);
+}
+
+__device__ __forceinline__ void raise_abort(AttnSmem& sm, int* status, int site) {
+  report_status(status, kStatusTimeout, site);
+  sm.abort = 1;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                     const __grid_constant__ CUtensorMap tm_v, const __nv_bfloat16* __restrict__ k_seedmask,
+                     const __nv_bfloat16* __restrict__ v_seedmask, const int32_t* __restrict__ seed_idx, int n_seeds,
+                     int Hq, int Hkv, int L, int n_mblk, float scale_log2, __nv_bfloat16* __restrict__ out,
+                     float* __restrict__ lse, int* status) {
+  extern __shared__ uint8_t smem_raw[];
+  AttnSmem& sm = *reinterpret_cast<AttnSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
+  const int mblk = blockIdx.x % n_mblk;
+  const int hq = (blockIdx.x / n_mblk) % Hq;
+  const int b = blockIdx.x / (n_mblk * Hq);
+  const int hkv = hq / (Hq / Hkv);
+  const int row0 = mblk * kRowsPerCta;
+  const int nkv = (L + kBN - 1) / kBN;
+  const int tail_valid = L - (nkv - 1) * kBN;   // valid keys in the last KV tile (1..128)
+
+  // ---------------- prologue ----------------
+  if (tid == 0) {
+    mbar_init(&sm.bar_q, 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&sm.bar_k_full[s], 1);
+      mbar_init(&sm.bar_k_empty[s], 1);
+      mbar_init(&sm.bar_v_full[s], 1);
+      mbar_init(&sm.bar_v_empty[s], 1);
+    }
+    for (int t = 0; t < kNQ; ++t) {
+      mbar_init(&sm.bar_s_full[t], 1);
+      mbar_init(&sm.bar_p_full[t], kBM);
+      mbar_init(&sm.bar_o_full[t], 1);
+    }
+    mbar_init(&sm.bar_drain, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  route_clear(sm.slot, kRowsPerCta, tid, kThreads);
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  route_scan(sm.slot, seed_idx + static_cast<size_t>(b) * n_seeds, n_seeds, row0, kRowsPerCta, L, tid, kThreads);
+  __syncthreads();
+  const uint32_t tbase = sm.tmem_base;
+
+  if (warp == kTmaWarp) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      mbar_arrive_expect_tx(&sm.bar_q, kNQ * kTileBytes);
+      for (int t = 0; t < kNQ; ++t)
+        for (int h = 0; h < 2; ++h)
+          tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q, 64 * h, row0 + t * kBM, hq, b);
+      int last_kj = -1, last_vj = -1;   // last KV tiles whose K / V loads were issued
+      bool ok = true;
+      for (int j = 0; j < nkv && ok; ++j) {
+        const int st = j & 1, n = j >> 1;
+        if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(&sm.bar_k_full[st], kTileBytes);
+        for (int h = 0; h < 2; ++h)
+          tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, j * kBN, hkv, b);
+        last_kj = j;
+        if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(&sm.bar_v_full[st], kTileBytes);
+        for (int h = 0; h < 2; ++h)
+          tma_load_4d(sm.v[st] + h * kBoxBytes, &tm_v, &sm.bar_v_full[st], 64 * h, j * kBN, hkv, b);
+        last_vj = j;
+      }
+      if (!ok) {
+        raise_abort(sm, status, 10);
+        // let every copy already issued land before the CTA's shared memory is released
+        mbar_wait(&sm.bar_q, 0, nullptr);
+        for (int jj = max(0, last_kj - 1); jj <= last_kj; ++jj)
+          mbar_wait(&sm.bar_k_full[jj & 1], (jj >> 1) & 1, nullptr);
+        for (int jj = max(0, last_vj - 1); jj <= last_vj; ++jj)
+          mbar_wait(&sm.bar_v_full[jj & 1], (jj >> 1) & 1, nullptr);
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      constexpr uint32_t id_qk = idesc_bf16_f32(kBM, kBN, false, false);
+      constexpr uint32_t id_pv = idesc_bf16_f32(kBM, kD, false, true);
+      bool ok = mbar_wait(&sm.bar_q, 0, &sm.abort);
+      tc_fence_after_sync();
+      // descriptors of stage / tile 0; the others are one tile (kTileBytes >> 4 units) further
+      constexpr uint64_t kTileDesc = kTileBytes >> 4;
+      const uint64_t dq0 = sdesc_sw128(smem_u32(sm.q[0]), 16, 1024);
+      const uint64_t dk0 = sdesc_sw128(smem_u32(sm.k[0]), 16, 1024);
+      const uint64_t dv0 = sdesc_sw128(smem_u32(sm.v[0]), kBoxBytes, 1024);
+      for (int j = 0; j <= nkv && ok; ++j) {
+        const int st = j & 1;
+        if (j < nkv) {
+          ok = mbar_wait(&sm.bar_k_full[st], (j >> 1) & 1, &sm.abort);
+          if (!ok) break;
+        }
+        if (j > 0) {
+          const int pst = (j - 1) & 1;
+          ok = mbar_wait(&sm.bar_v_full[pst], ((j - 1) >> 1) & 1, &sm.abort);
+          if (!ok) break;
+        }
+        tc_fence_after_sync();
+        for (int t = 0; t < kNQ && ok; ++t) {
+          if (j > 0) {
+            // O_t += P_t(j-1) . V(j-1); P from tensor memory, V MN-major from shared memory
+            ok = mbar_wait(&sm.bar_p_full[t], (j - 1) & 1, &sm.abort);
+            if (!ok) break;
+            tc_fence_after_sync();
+            const int pst = (j - 1) & 1;
+#pragma unroll
+            for (int ks = 0; ks < kBN / 16; ++ks)
+              umma_ts(tbase + col_o(t), tbase + col_s(t) + 8 * ks,
+                      dv0 + pst * kTileDesc + static_cast<uint64_t>((ks * 2048) >> 4),
+                      id_pv, (j > 1 || ks > 0) ? 1u : 0u);
+            if (j == nkv) umma_commit(&sm.bar_o_full[t]);
+          }
+          if (j < nkv) {
+            // S_t = Q_t . K(j)^T, both K-major with 128-byte swizzle
+#pragma unroll
+            for (int ks = 0; ks < kD / 16; ++ks) {
+              const uint64_t off = static_cast<uint64_t>(((ks >> 2) * kBoxBytes + (ks & 3) * 32) >> 4);
+              umma_ss(tbase + col_s(t), dq0 + t * kTileDesc + off, dk0 + st * kTileDesc + off, id_qk,
+                      ks > 0 ? 1u : 0u);
+            }
+            umma_commit(&sm.bar_s_full[t]);
+          }
+        }
+        if (!ok) break;
+        if (j < nkv) umma_commit(&sm.bar_k_empty[st]);
+        if (j > 0) umma_commit(&sm.bar_v_empty[(j - 1) & 1]);
+      }
+      if (!ok) raise_abort(sm, status, 20);
+      // all tensor-core work of this CTA must finish before tensor memory is released
+      umma_commit(&sm.bar_drain);
+      mbar_wait(&sm.bar_drain, 0, nullptr);
+    }
+  } else {
+    // ---------------- softmax (warps 0-7) ----------------
+    const int qt = warp >> 2;
+    const int r = tid & (kBM - 1);
+    const uint32_t trow = tbase + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+    const uint32_t s_addr = trow + col_s(qt);
+    const uint32_t o_addr = trow + col_o(qt);
+    const int grow = row0 + qt * kBM + r;
+    const int my_slot = sm.slot[qt * kBM + r];
+    const bool is_seed = my_slot != kNoSlot;
+    const int diag_j = (row0 + qt * kBM) / kBN;
+    float m_run = -INFINITY, l_run = 0.0f;
+    bool ok = true;
+
+    for (int j = 0; j < nkv; ++j) {
+      ok = warp_wait(&sm.bar_s_full[qt], j & 1, &sm.abort);
+      if (!ok) break;
+      tc_fence_after_sync();
+      uint32_t raw[4][32];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(s_addr + 32 * c, raw[c]);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld_wait(raw[c]);
+      float* s = reinterpret_cast<float*>(&raw[0][0]);
+      if (j == nkv - 1 && tail_valid < kBN) {
+#pragma unroll
+        for (int c = 0; c < kBN; ++c)
+          if (c >= tail_valid) s[c] = -INFINITY;
+      }
+      if (j == diag_j && __any_sync(0xffffffffu, is_seed)) {
+        // exclusion of the cached diagonal term of a seed row
+#pragma unroll
+        for (int c = 0; c < kBN; ++c)
+          if (is_seed && c == r) s[c] = -INFINITY;
+      }
+      float mx = s[0];
+#pragma unroll
+      for (int c = 1; c < kBN; ++c) mx = fmaxf(mx, s[c]);
+      const float m_tile = mx * scale_log2;
+      float alpha = 1.0f;
+      bool rescaled = false;
+      if (m_tile > m_run + kRescaleThreshold) {
+        alpha = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m_tile);
+        m_run = m_tile;
+        rescaled = true;
+      }
+      const float m_use = (m_run == -INFINITY) ? 0.0f : m_run;
+      uint32_t packed[64];
+      float rowsum = 0.0f;
+#pragma unroll
+      for (int c = 0; c < 64; ++c) {
+        const float p0 = ex2_approx(fmaf(s[2 * c], scale_log2, -m_use));
+        const float p1 = ex2_approx(fmaf(s[2 * c + 1], scale_log2, -m_use));
+        rowsum += p0 + p1;
+        packed[c] = pack_bf16x2(p0, p1);
+      }
+      l_run = l_run * alpha + rowsum;
+      tmem_st32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&packed[0]));
+      tmem_st32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&packed[32]));
+      if (j > 0 && __any_sync(0xffffffffu, rescaled)) {
+        // O holds the products of tiles < j (complete: they were issued before S(j))
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[32];
+          tmem_ld32(o_addr + 32 * c, o);
+          tmem_ld_wait(o);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+          tmem_st32(o_addr + 32 * c, o);
+        }
+      }
+      tmem_st_wait();
+      tc_fence_before_sync();
+      mbar_arrive(&sm.bar_p_full[qt]);
+    }
+    if (ok) ok = warp_wait(&sm.bar_o_full[qt], 0, &sm.abort);
+    if (ok) ok = warp_wait(&sm.bar_q, 0, &sm.abort);
+    if (!ok) {
+      if (!sm.abort) raise_abort(sm, status, 30 + qt);
+    } else {
+      tc_fence_after_sync();
+      uint32_t oraw[4][32];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(o_addr + 32 * c, oraw[c]);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld_wait(oraw[c]);
+      float* o = reinterpret_cast<float*>(&oraw[0][0]);
+      if (is_seed) {
+        // merge the masked-input self term (k_i, v_i) of this seed row
+        const size_t mrow = ((static_cast<size_t>(b) * Hkv + hkv) * n_seeds + my_slot) * kD;
+        const uint4* kmv = reinterpret_cast<const uint4*>(k_seedmask + mrow);
+        const uint4* vmv = reinterpret_cast<const uint4*>(v_seedmask + mrow);
+        float dot = 0.0f;
+#pragma unroll
+        for (int ch = 0; ch < 16; ++ch) {
+          const int h = ch >> 3, c8 = ch & 7;
+          const uint4 qv = *reinterpret_cast<const uint4*>(sm.q[qt] + h * kBoxBytes + r * 128 +
+                                                           ((c8 ^ (r & 7)) * 16));
+          const uint4 kv = __ldg(kmv + ch);
+          const __nv_bfloat162* qp = reinterpret_cast<const __nv_bfloat162*>(&qv);
+          const __nv_bfloat162* kp = reinterpret_cast<const __nv_bfloat162*>(&kv);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 qf = __bfloat1622float2(qp[e]);
+            const float2 kf = __bfloat1622float2(kp[e]);
+            dot = fmaf(qf.x, kf.x, dot);
+            dot = fmaf(qf.y, kf.y, dot);
+          }
+        }
+        const float s_self = dot * scale_log2;
+        const float m2 = fmaxf(m_run, s_self);
+        const float a = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m2);
+        const float pself = ex2_approx(s_self - m2);
+        l_run = l_run * a + pself;
+#pragma unroll
+        for (int ch = 0; ch < 16; ++ch) {
+          const uint4 vv = __ldg(vmv + ch);
+          const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 vf = __bfloat1622float2(vp[e]);
+            o[ch * 8 + 2 * e] = o[ch * 8 + 2 * e] * a + pself * vf.x;
+            o[ch * 8 + 2 * e + 1] = o[ch * 8 + 2 * e + 1] * a + pself * vf.y;
+          }
+        }
+        m_run = m2;
+      }
+      if (grow < L) {
+        const float inv = 1.0f / l_run;
+        uint4* dst = reinterpret_cast<uint4*>(out + ((static_cast<size_t>(b) * Hq + hq) * L + grow) * kD);
+#pragma unroll
+        for (int ch = 0; ch < 16; ++ch) {
+          uint4 w;
+          w.x = pack_bf16x2(o[ch * 8 + 0] * inv, o[ch * 8 + 1] * inv);
+          w.y = pack_bf16x2(o[ch * 8 + 2] * inv, o[ch * 8 + 3] * inv);
+          w.z = pack_bf16x2(o[ch * 8 + 4] * inv, o[ch * 8 + 5] * inv);
+          w.w = pack_bf16x2(o[ch * 8 + 6] * inv, o[ch * 8 + 7] * inv);
+          dst[ch] = w;
+        }
+        if (lse != nullptr)
+          lse[(static_cast<size_t>(b) * Hq + hq) * L + grow] = (m_run + log2f(l_run)) * 0.6931471805599453f;
+      }
+    }
+  }
+
+  // ---------------- teardown ----------------
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  if (warp == kMmaWarp) tmem_dealloc(tbase, 512);
+}
+
+}  // namespace
+
+int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) {
+  CUtensorMap tq, tk, tv;
+  if (!make_bf16_map_4d(&tq, a.q, kD, a.L, a.Hq, a.B, kBM) ||
+      !make_bf16_map_4d(&tk, a.k_cached, kD, a.L, a.Hkv, a.B, kBN) ||
+      !make_bf16_map_4d(&tv, a.v_cached, kD, a.L, a.Hkv, a.B, kBN))
+    return -3;
+  const int n_mblk = (a.L + kRowsPerCta - 1) / kRowsPerCta;
+  const long long grid = static_cast<long long>(n_mblk) * a.Hq * a.B;
+  if (grid > 0x7fffffffLL) return -2;
+  const size_t smem = sizeof(AttnSmem) + 1024;
+  static bool attr_set = false;
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(attn_bf16_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
+        cudaSuccess)
+      return -3;
+    attr_set = true;
+  }
+  const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
+  attn_bf16_kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
+      tq, tk, tv, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
+      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.L, n_mblk, scale_log2, static_cast<__nv_bfloat16*>(a.out), a.lse,
+      status);
+  return cudaGetLastError() == cudaSuccess ? 0 : -3;
+}
+
+}  // namespace cover

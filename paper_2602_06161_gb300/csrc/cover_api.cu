@@ -1,0 +1,159 @@
+// cover_api.cu - the extern "C" entry points declared in include/cover.h and
+// include/cover_debug.h: argument validation, the per-device status block,
+// and dispatch to the kernel launchers.
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "cover.h"
+#include "cover_debug.h"
+#include "kernels.cuh"
+
+namespace {
+
+// Per-device status block written by kernels that give up on a bounded wait:
+// [0] status code, [1] site id, [2] block id, [3] unused.
+__device__ int g_status[4];
+
+constexpr int kMaxDevices = 64;
+int* g_status_addr[kMaxDevices];
+std::mutex g_status_mu;
+
+int* status_block() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_status_mu);
+  if (g_status_addr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
+    g_status_addr[dev] = static_cast<int*>(p);
+  }
+  return g_status_addr[dev];
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int check_attn_args(const void* q, const void* kc, const void* vc, const void* km, const void* vm,
+                    const int32_t* seed_idx, int n_seeds, int B, int Hq, int Hkv, int L, int D, const void* out,
+                    const float* lse, size_t align) {
+  if (q == nullptr || kc == nullptr || vc == nullptr || out == nullptr) return COVER_ERR_INVALID_ARG;
+  if (B < 1 || Hq < 1 || Hkv < 1 || L < 1 || D < 1) return COVER_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0) return COVER_ERR_INVALID_ARG;
+  if (n_seeds < 0 || n_seeds > L) return COVER_ERR_INVALID_ARG;
+  if (n_seeds > 0 && (seed_idx == nullptr || km == nullptr || vm == nullptr)) return COVER_ERR_INVALID_ARG;
+  if (!aligned(q, align) || !aligned(kc, align) || !aligned(vc, align) || !aligned(out, align))
+    return COVER_ERR_INVALID_ARG;
+  if (n_seeds > 0 && (!aligned(km, align) || !aligned(vm, align) || !aligned(seed_idx, 4)))
+    return COVER_ERR_INVALID_ARG;
+  if (lse != nullptr && !aligned(lse, 4)) return COVER_ERR_INVALID_ARG;
+  return COVER_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int cover_attn_fwd(const void* q, const void* k_cached, const void* v_cached, const void* k_seedmask,
+                   const void* v_seedmask, const int32_t* seed_idx, int n_seeds, int B, int Hq, int Hkv, int L, int D,
+                   void* out, float* lse, void* stream) {
+  int rc = check_attn_args(q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, L, D, out,
+                           lse, 16);
+  if (rc != COVER_OK) return rc;
+  if (D != 128) return COVER_ERR_UNSUPPORTED;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, L, D, out, lse};
+  return cover::launch_attn_bf16_sm103(a, st, static_cast<cudaStream_t>(stream));
+}
+
+int cover_attn_fwd_f32(const float* q, const float* k_cached, const float* v_cached, const float* k_seedmask,
+                       const float* v_seedmask, const int32_t* seed_idx, int n_seeds, int B, int Hq, int Hkv, int L,
+                       int D, float* out, float* lse, void* stream) {
+  int rc = check_attn_args(q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, L, D, out,
+                           lse, 4);
+  if (rc != COVER_OK) return rc;
+  if (D != 64 && D != 128) return COVER_ERR_UNSUPPORTED;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, L, D, out, lse};
+  return cover::launch_attn_f32(a, st, static_cast<cudaStream_t>(stream));
+}
+
+int cover_seed_route(const int32_t* seed_idx, int n_seeds, int B, int L, int32_t* slot_out, uint32_t* bitmap_out,
+                     int32_t* n_invalid_out, void* stream) {
+  if (B < 1 || L < 1 || n_seeds < 0 || n_seeds > L) return COVER_ERR_INVALID_ARG;
+  if (n_seeds > 0 && seed_idx == nullptr) return COVER_ERR_INVALID_ARG;
+  if (slot_out == nullptr || bitmap_out == nullptr || n_invalid_out == nullptr) return COVER_ERR_INVALID_ARG;
+  if (B > 65535) return COVER_ERR_UNSUPPORTED;
+  return cover::launch_seed_route(seed_idx, n_seeds, B, L, slot_out, bitmap_out, n_invalid_out,
+                                  static_cast<cudaStream_t>(stream));
+}
+
+size_t cover_score_workspace_bytes(int n_seq) { return n_seq > 0 ? sizeof(uint32_t) * static_cast<size_t>(n_seq) : 0; }
+
+int cover_score_fwd(const void* logits, int N, int V, int n_seq, const int32_t* cur_tok, const float* d_in,
+                    const float* d_out, const uint8_t* eligible, int topk, float* maxprob, float* entropy,
+                    int32_t* argmax, float* score, int32_t* topk_idx, float* topk_score, void* workspace,
+                    void* stream) {
+  if (logits == nullptr || maxprob == nullptr || entropy == nullptr || argmax == nullptr || score == nullptr)
+    return COVER_ERR_INVALID_ARG;
+  if (N < 1 || V < 1 || n_seq < 1 || N % n_seq != 0) return COVER_ERR_INVALID_ARG;
+  const int per = N / n_seq;
+  if (per > 4096) return COVER_ERR_INVALID_ARG;
+  if (topk < 0 || topk > per) return COVER_ERR_INVALID_ARG;
+  if (topk > 0 && (topk_idx == nullptr || workspace == nullptr)) return COVER_ERR_INVALID_ARG;
+  if (!aligned(logits, 16) || !aligned(maxprob, 4) || !aligned(entropy, 4) || !aligned(argmax, 4) ||
+      !aligned(score, 4))
+    return COVER_ERR_INVALID_ARG;
+  if (workspace != nullptr && !aligned(workspace, 4)) return COVER_ERR_INVALID_ARG;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  cover::ScoreArgs a{logits, N, V, n_seq, cur_tok, d_in, d_out, eligible, topk, maxprob, entropy, argmax,
+                     score, topk_idx, topk_score, static_cast<uint32_t*>(workspace)};
+  return cover::launch_score(a, st, static_cast<cudaStream_t>(stream));
+}
+
+int cover_device_status(void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return COVER_ERR_CUDA;
+  int host[4] = {0, 0, 0, 0};
+  if (cudaMemcpyAsync(host, st, sizeof(host), cudaMemcpyDeviceToHost, s) != cudaSuccess) return COVER_ERR_CUDA;
+  if (cudaMemsetAsync(st, 0, sizeof(host), s) != cudaSuccess) return COVER_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return COVER_ERR_CUDA;
+  return host[0];
+}
+
+const char* cover_status_str(int code) {
+  switch (code) {
+    case COVER_OK: return "COVER_OK";
+    case COVER_ERR_INVALID_ARG: return "COVER_ERR_INVALID_ARG";
+    case COVER_ERR_UNSUPPORTED: return "COVER_ERR_UNSUPPORTED";
+    case COVER_ERR_CUDA: return "COVER_ERR_CUDA";
+    case COVER_ERR_DEVICE_TIMEOUT: return "COVER_ERR_DEVICE_TIMEOUT";
+    default: return "COVER_ERR_UNKNOWN";
+  }
+}
+
+int cover_debug_umma_tile(const void* a, const void* b, const void* p, const void* v, float* c1, float* c2,
+                          void* stream) {
+  if (a == nullptr || b == nullptr || p == nullptr || v == nullptr || c1 == nullptr || c2 == nullptr)
+    return COVER_ERR_INVALID_ARG;
+  if (!aligned(a, 16) || !aligned(b, 16) || !aligned(p, 16) || !aligned(v, 16) || !aligned(c1, 16) ||
+      !aligned(c2, 16))
+    return COVER_ERR_INVALID_ARG;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  return cover::launch_umma_tile(a, b, p, v, c1, c2, st, static_cast<cudaStream_t>(stream));
+}
+
+int cover_debug_wait_timeout(int limit_us, void* stream) {
+  if (limit_us < 1 || limit_us > 2000000) return COVER_ERR_INVALID_ARG;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  return cover::launch_wait_timeout(static_cast<uint64_t>(limit_us) * 1000ull, st,
+                                    static_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

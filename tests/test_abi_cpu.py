@@ -1,0 +1,102 @@
+"""CPU checks of the C-ABI library: it builds, loads without a GPU, exports every
+declared symbol, and rejects invalid arguments before touching CUDA."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2602_06161_gb300 import _lib, build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = []
+    for h in sorted(os.listdir(os.path.join(ROOT, "include"))):
+        if h.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", h)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names += re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\**\s*(cover_[A-Za-z0-9_]+)\s*\(",
+                                text, flags=re.M)
+    return names
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return _lib.load()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 9
+    raw = ctypes.CDLL(build.LIB)
+    for n in names:
+        assert hasattr(raw, n), n
+    assert sorted(names) == sorted(_lib.exported_symbols())
+
+
+def test_status_strings(lib):
+    assert _lib.status_str(0) == "COVER_OK"
+    assert _lib.status_str(-1) == "COVER_ERR_INVALID_ARG"
+    assert _lib.status_str(-4) == "COVER_ERR_DEVICE_TIMEOUT"
+    assert _lib.status_str(12345) == "COVER_ERR_UNKNOWN"
+
+
+# fake, 16-byte aligned, never dereferenced (argument checks return first)
+P = 0x10000
+
+
+def attn(lib, **kw):
+    a = dict(q=P, kc=P, vc=P, km=P, vm=P, seeds=P, S=2, B=1, Hq=2, Hkv=1, L=128, D=128, out=P, lse=P)
+    a.update(kw)
+    return lib.cover_attn_fwd(a["q"], a["kc"], a["vc"], a["km"], a["vm"], a["seeds"], a["S"], a["B"], a["Hq"],
+                              a["Hkv"], a["L"], a["D"], a["out"], a["lse"], None)
+
+
+@pytest.mark.parametrize("kw", [
+    dict(q=None), dict(out=None), dict(kc=None), dict(B=0), dict(L=0), dict(Hq=3, Hkv=2), dict(Hkv=0),
+    dict(S=-1), dict(S=129), dict(seeds=None), dict(km=None), dict(q=P + 8), dict(out=P + 2), dict(lse=P + 2),
+    dict(D=0),
+])
+def test_attn_invalid_args(lib, kw):
+    assert attn(lib, **kw) == -1
+
+
+def test_attn_unsupported_head_dim(lib):
+    assert attn(lib, D=64) == -2
+    assert attn(lib, D=96) == -2
+
+
+def score(lib, **kw):
+    a = dict(logits=P, N=8, V=16, n_seq=2, k=2, mp=P, ent=P, am=P, sc=P, ti=P, ts=P, ws=P)
+    a.update(kw)
+    return lib.cover_score_fwd(a["logits"], a["N"], a["V"], a["n_seq"], None, None, None, None, a["k"], a["mp"],
+                               a["ent"], a["am"], a["sc"], a["ti"], a["ts"], a["ws"], None)
+
+
+@pytest.mark.parametrize("kw", [
+    dict(logits=None), dict(N=0), dict(V=0), dict(n_seq=3), dict(n_seq=0), dict(k=5), dict(k=-1),
+    dict(ti=None), dict(ws=None), dict(logits=P + 2), dict(mp=None), dict(N=2 * 4097, n_seq=2),
+])
+def test_score_invalid_args(lib, kw):
+    assert score(lib, **kw) == -1
+
+
+def test_route_invalid_args(lib):
+    assert lib.cover_seed_route(P, 2, 0, 10, P, P, P, None) == -1
+    assert lib.cover_seed_route(P, 11, 1, 10, P, P, P, None) == -1
+    assert lib.cover_seed_route(None, 2, 1, 10, P, P, P, None) == -1
+    assert lib.cover_seed_route(P, 2, 1, 10, None, P, P, None) == -1
+
+
+def test_debug_invalid_args(lib):
+    assert lib.cover_debug_wait_timeout(0, None) == -1
+    assert lib.cover_debug_wait_timeout(3000000, None) == -1
+    assert lib.cover_debug_umma_tile(None, P, P, P, P, P, None) == -1
+
+
+def test_workspace_bytes(lib):
+    assert lib.cover_score_workspace_bytes(8) == 32
+    assert lib.cover_score_workspace_bytes(0) == 0
