@@ -167,14 +167,19 @@ def test_bf16_invariances_bit_exact():
     inp = W.make_attn_inputs(2, 4, 2, 640, 128, 24, dtype="bf16", seed=21)
     args = _dev_inputs(inp)
     out0, lse0 = api.cover_attn_fwd(*args)
-    # perturb every seed's own cached pair: seed rows must not change at all
-    kc, vc = args[1].clone(), args[2].clone()
-    for b in range(2):
-        for i in inp.seed_idx[b]:
-            kc[b, :, i] = kc[b, :, i] * 3 + 1
-            vc[b, :, i] = -vc[b, :, i] + 2
-    out1, lse1 = api.cover_attn_fwd(args[0], kc, vc, *args[3:])
-    # perturb the masked buffer: non-seed rows must not change at all
+    # a seed row must not change at all when its own cached pair changes (other rows do see it)
+    for b, s in [(0, 0), (0, 5), (1, 11), (1, 23)]:
+        i = int(inp.seed_idx[b, s])
+        kc, vc = args[1].clone(), args[2].clone()
+        kc[b, :, i] = kc[b, :, i] * 3 + 1
+        vc[b, :, i] = -vc[b, :, i] + 2
+        out1, lse1 = api.cover_attn_fwd(args[0], kc, vc, *args[3:])
+        torch.cuda.synchronize()
+        assert torch.equal(out0[b, :, i], out1[b, :, i])
+        assert torch.equal(lse0[b, :, i], lse1[b, :, i])
+        j = (i + 1) % 640
+        assert not torch.equal(out0[b, :, j], out1[b, :, j])
+    # non-seed rows must not change at all when the masked buffer changes
     out2, lse2 = api.cover_attn_fwd(*args[:3], args[3] * 5 - 1, args[4] + 3, args[5])
     torch.cuda.synchronize()
     seed_mask = np.zeros((2, 640), bool)
@@ -182,11 +187,8 @@ def test_bf16_invariances_bit_exact():
         seed_mask[b, inp.seed_idx[b]] = True
     sm = torch.from_numpy(seed_mask).cuda()
     for b in range(2):
-        assert torch.equal(out0[b][:, sm[b]], out1[b][:, sm[b]])
-        assert torch.equal(lse0[b][:, sm[b]], lse1[b][:, sm[b]])
         assert torch.equal(out0[b][:, ~sm[b]], out2[b][:, ~sm[b]])
         assert torch.equal(lse0[b][:, ~sm[b]], lse2[b][:, ~sm[b]])
-        assert not torch.equal(out0[b][:, ~sm[b]], out1[b][:, ~sm[b]])
         assert not torch.equal(out0[b][:, sm[b]], out2[b][:, sm[b]])
 
 
