@@ -241,7 +241,38 @@ __global__ void __launch_bounds__(kThreads, 1)
     float m_run = -INFINITY, l_run = 0.0f;
     bool ok = true;
 
-    for (int j = 0; j < nkv; ++j) {
+    // Seed rows: score of the masked-input self pair, s_self = q_i . k_i (log2-scaled),
+    // computed up front so its global loads overlap the first tiles; the value row
+    // is prefetched into L2 for the epilogue.
+    float s_self = 0.0f;
+    const size_t mrow = is_seed ? ((static_cast<size_t>(b) * Hkv + hkv) * n_seeds + my_slot) * kD : 0;
+    if (__any_sync(0xffffffffu, is_seed)) {
+      ok = warp_wait(&sm.bar_q, 0, &sm.abort);
+      if (ok && is_seed) {
+        prefetch_l2(v_seedmask + mrow);
+        prefetch_l2(v_seedmask + mrow + 64);
+        const uint4* kmv = reinterpret_cast<const uint4*>(k_seedmask + mrow);
+        float dot[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+        for (int ch = 0; ch < 16; ++ch) {
+          const int h = ch >> 3, c8 = ch & 7;
+          const uint4 qv = *reinterpret_cast<const uint4*>(sm.q[qt] + h * kBoxBytes + r * 128 + ((c8 ^ (r & 7)) * 16));
+          const uint4 kv = __ldg(kmv + ch);
+          const __nv_bfloat162* qp = reinterpret_cast<const __nv_bfloat162*>(&qv);
+          const __nv_bfloat162* kp = reinterpret_cast<const __nv_bfloat162*>(&kv);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 qf = __bfloat1622float2(qp[e]);
+            const float2 kf = __bfloat1622float2(kp[e]);
+            dot[e] = fmaf(qf.x, kf.x, dot[e]);
+            dot[e] = fmaf(qf.y, kf.y, dot[e]);
+          }
+        }
+        s_self = ((dot[0] + dot[1]) + (dot[2] + dot[3])) * scale_log2;
+      }
+    }
+
+    for (int j = 0; j < nkv && ok; ++j) {
       ok = warp_wait(&sm.bar_s_full[qt], j & 1, &sm.abort);
       if (!ok) break;
       tc_fence_after_sync();
@@ -262,10 +293,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < kBN; ++c)
           if (is_seed && c == r) s[c] = -INFINITY;
       }
-      float mx = s[0];
+      // row maximum: four independent 3-input max chains
+      float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
 #pragma unroll
-      for (int c = 1; c < kBN; ++c) mx = fmaxf(mx, s[c]);
-      const float m_tile = mx * scale_log2;
+      for (int c = 4; c < kBN; c += 8) {
+        mx0 = fmax3(mx0, s[c], s[c + 1]);
+        mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
+        mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
+        mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
+      }
+      const float m_tile = fmax3(mx0, mx1, fmaxf(mx2, mx3)) * scale_log2;
       float alpha = 1.0f;
       bool rescaled = false;
       if (m_tile > m_run + kRescaleThreshold) {
@@ -274,15 +311,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         rescaled = true;
       }
       const float m_use = (m_run == -INFINITY) ? 0.0f : m_run;
+      // p = 2^(s * scale - m) on pairs; four independent partial row sums
+      const uint64_t scale2 = f2_pack(scale_log2, scale_log2);
+      const uint64_t negm2 = f2_pack(-m_use, -m_use);
+      uint64_t acc2[4] = {0, 0, 0, 0};
       uint32_t packed[64];
-      float rowsum = 0.0f;
 #pragma unroll
       for (int c = 0; c < 64; ++c) {
-        const float p0 = ex2_approx(fmaf(s[2 * c], scale_log2, -m_use));
-        const float p1 = ex2_approx(fmaf(s[2 * c + 1], scale_log2, -m_use));
-        rowsum += p0 + p1;
+        float t0, t1;
+        f2_unpack(f2_fma(f2_pack(s[2 * c], s[2 * c + 1]), scale2, negm2), t0, t1);
+        const float p0 = ex2_approx(t0);
+        const float p1 = ex2_approx(t1);
         packed[c] = pack_bf16x2(p0, p1);
+        acc2[c & 3] = f2_add(acc2[c & 3], f2_pack(p0, p1));
       }
+      float rs[8];
+      f2_unpack(f2_add(acc2[0], acc2[1]), rs[0], rs[1]);
+      f2_unpack(f2_add(acc2[2], acc2[3]), rs[2], rs[3]);
+      const float rowsum = (rs[0] + rs[1]) + (rs[2] + rs[3]);
       l_run = l_run * alpha + rowsum;
       tmem_st32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&packed[0]));
       tmem_st32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&packed[32]));
@@ -316,27 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       float* o = reinterpret_cast<float*>(&oraw[0][0]);
       if (is_seed) {
         // merge the masked-input self term (k_i, v_i) of this seed row
-        const size_t mrow = ((static_cast<size_t>(b) * Hkv + hkv) * n_seeds + my_slot) * kD;
-        const uint4* kmv = reinterpret_cast<const uint4*>(k_seedmask + mrow);
         const uint4* vmv = reinterpret_cast<const uint4*>(v_seedmask + mrow);
-        float dot = 0.0f;
-#pragma unroll
-        for (int ch = 0; ch < 16; ++ch) {
-          const int h = ch >> 3, c8 = ch & 7;
-          const uint4 qv = *reinterpret_cast<const uint4*>(sm.q[qt] + h * kBoxBytes + r * 128 +
-                                                           ((c8 ^ (r & 7)) * 16));
-          const uint4 kv = __ldg(kmv + ch);
-          const __nv_bfloat162* qp = reinterpret_cast<const __nv_bfloat162*>(&qv);
-          const __nv_bfloat162* kp = reinterpret_cast<const __nv_bfloat162*>(&kv);
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 qf = __bfloat1622float2(qp[e]);
-            const float2 kf = __bfloat1622float2(kp[e]);
-            dot = fmaf(qf.x, kf.x, dot);
-            dot = fmaf(qf.y, kf.y, dot);
-          }
-        }
-        const float s_self = dot * scale_log2;
         const float m2 = fmaxf(m_run, s_self);
         const float a = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m2);
         const float pself = ex2_approx(s_self - m2);
