@@ -76,6 +76,11 @@ def max_over_ranks(x: float, ws: int) -> float:
     return float(t.item())
 
 
+def weak_scaling_value(flops_per_rank: float, ms_per_step_max: float, ws: int) -> float:
+    """Whole-job TFLOP/s: every rank processes its own replica of the workload."""
+    return ws * flops_per_rank / (ms_per_step_max * 1e-3) / 1e12
+
+
 def barrier(ws: int):
     if ws > 1:
         import torch.distributed as dist
@@ -269,7 +274,7 @@ def run_ours(args):
     attn_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_attn)
     score_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_score)
     flops = wl.attn_flops
-    value = ws * flops / (ms_step * 1e-3) / 1e12
+    value = weak_scaling_value(flops, ms_step, ws)
 
     peaks, peak_kind = load_peaks()
     timed_s = ms_total / 1e3
