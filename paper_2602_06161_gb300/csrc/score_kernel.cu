@@ -15,8 +15,18 @@
 // with a self-resetting atomicInc counter per segment - sorts the segment's
 // eligible rows by (score descending, index ascending) with a bitonic sort of
 // 64-bit keys in shared memory and writes the first k.
+//
+// Two ways to stream a row:
+//  * score_bulk_kernel (rows 16-byte aligned, V % 8 == 0): a producer warp
+//    issues cp.async.bulk copies of 8 KB chunks into a 6-stage shared-memory
+//    ring (mbarrier full / empty), 8 consumer warps reduce from shared memory;
+//    bytes in flight do not cost registers, and 4 CTAs share an SM.
+//  * score_kernel (any V): 16-byte non-allocating global loads, scalar head and
+//    tail for rows that do not start on a 16-byte boundary.
 #include <math.h>
 #include <stdint.h>
+
+#include <algorithm>
 
 #include "kernels.cuh"
 #include "ptx.cuh"
@@ -24,9 +34,14 @@
 namespace cover {
 namespace {
 
-constexpr int kThreads = 512;
+constexpr int kThreads = 512;              // register-load kernel
 constexpr int kWarps = kThreads / 32;
 constexpr int kUnroll = 4;
+constexpr int kConsumerWarps = 8;          // bulk kernel: consumers + 1 producer warp
+constexpr int kBulkThreads = (kConsumerWarps + 1) * 32;
+constexpr int kChunkElems = 4096;          // 8 KB of bf16 per bulk copy
+constexpr int kChunkBytes = kChunkElems * 2;
+constexpr int kRingStages = 6;
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct RowAcc {
@@ -112,76 +127,20 @@ __device__ __forceinline__ float order_key_inv(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
 }
 
-__global__ void __launch_bounds__(kThreads, 2)
-    score_kernel(const uint16_t* __restrict__ logits, int V, int per_seq, const int32_t* __restrict__ cur_tok,
-                 const float* __restrict__ d_in, const float* __restrict__ d_out,
-                 const uint8_t* __restrict__ eligible, int topk, int sort_n, float* __restrict__ maxprob,
-                 float* __restrict__ entropy, int32_t* __restrict__ argmax, float* __restrict__ score,
-                 int32_t* __restrict__ topk_idx, float* __restrict__ topk_score, uint32_t* __restrict__ counters) {
-  extern __shared__ uint64_t keys[];
-  __shared__ float red_m[kWarps];
-  __shared__ int red_i[kWarps];
-  __shared__ double red_z[kWarps], red_s[kWarps];
-  __shared__ float s_max;
-  __shared__ int s_last;
 
-  const int n = blockIdx.x;
+// ---------------------------------------------------------------------------
+// per-row finish (all threads of the CTA call it; NW = warps in the CTA)
+// ---------------------------------------------------------------------------
+struct RowOut {
+  float M;      // row maximum
+  int yhat;     // first index attaining it
+  double Z, S;  // sum 2^t and sum t 2^t re-referenced to M log2(e)
+};
+
+template <int NW>
+__device__ __forceinline__ RowOut row_reduce(const RowAcc& a, float* red_m, int* red_i, double* red_z,
+                                             double* red_s) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const size_t row_off = static_cast<size_t>(n) * V;
-  const uint16_t* row = logits + row_off;
-
-  RowAcc a{-INFINITY, 0x7fffffff, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
-
-  // elements before the first 16-byte boundary of the row
-  const int head = min(static_cast<int>((8 - (row_off & 7)) & 7), V);
-  const int nvec = (V - head) / 8;
-  const int tail0 = head + nvec * 8;
-  if (tid < head) acc_scalar(a, bf16_to_f32(row[tid]), tid);
-
-  const uint4* vrow = reinterpret_cast<const uint4*>(row + head);
-  int v = tid;
-  for (; v + (kUnroll - 1) * kThreads < nvec; v += kUnroll * kThreads) {
-    uint4 w[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) w[u] = ld_stream(vrow + v + u * kThreads);
-    float x[kUnroll][8];
-    float bmax = -INFINITY;
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      unpack8(w[u], x[u]);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) bmax = fmaxf(bmax, x[u][k]);
-    }
-    if (bmax > a.m) {
-      int idx = 0x7fffffff;
-#pragma unroll
-      for (int u = kUnroll - 1; u >= 0; --u)
-#pragma unroll
-        for (int k = 7; k >= 0; --k)
-          if (x[u][k] == bmax) idx = head + (v + u * kThreads) * 8 + k;
-      raise_max(a, bmax, idx);
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) acc_vec8(a, x[u]);
-  }
-  for (; v < nvec; v += kThreads) {
-    float x[8];
-    unpack8(ld_stream(vrow + v), x);
-    float bmax = -INFINITY;
-#pragma unroll
-    for (int k = 0; k < 8; ++k) bmax = fmaxf(bmax, x[k]);
-    if (bmax > a.m) {
-      int idx = 0x7fffffff;
-#pragma unroll
-      for (int k = 7; k >= 0; --k)
-        if (x[k] == bmax) idx = head + v * 8 + k;
-      raise_max(a, bmax, idx);
-    }
-    acc_vec8(a, x);
-  }
-  if (tail0 + tid < V) acc_scalar(a, bf16_to_f32(row[tail0 + tid]), tail0 + tid);
-
-  // ---- row maximum and first index attaining it ----
   float m = a.m;
   int mi = a.mi;
 #pragma unroll
@@ -198,28 +157,18 @@ __global__ void __launch_bounds__(kThreads, 2)
     red_i[warp] = mi;
   }
   __syncthreads();
-  if (warp == 0) {
-    m = lane < kWarps ? red_m[lane] : -INFINITY;
-    mi = lane < kWarps ? red_i[lane] : 0x7fffffff;
+  float M = red_m[0];
+  int I = red_i[0];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
-      const int i2 = __shfl_xor_sync(0xffffffffu, mi, o);
-      if (m2 > m || (m2 == m && i2 < mi)) {
-        m = m2;
-        mi = i2;
-      }
-    }
-    if (lane == 0) {
-      s_max = m;
-      red_i[0] = mi;
+  for (int w = 1; w < NW; ++w) {
+    const float m2 = red_m[w];
+    const int i2 = red_i[w];
+    if (m2 > M || (m2 == M && i2 < I)) {
+      M = m2;
+      I = i2;
     }
   }
-  __syncthreads();
-  const float M = s_max;
   const float Mref = M * kLog2e;
-
-  // ---- partial sums re-referenced to the row maximum, summed in fp64 ----
   double zd = 0.0, sd = 0.0;
   if (a.m != -INFINITY) {
     const float d = a.mref - Mref;
@@ -239,44 +188,52 @@ __global__ void __launch_bounds__(kThreads, 2)
     red_s[warp] = sd;
   }
   __syncthreads();
+  RowOut r{M, I, 0.0, 0.0};
   if (tid == 0) {
-    double Z = 0.0, S = 0.0;
-    for (int w = 0; w < kWarps; ++w) {
-      Z += red_z[w];
-      S += red_s[w];
-    }
-    const int yhat = red_i[0];
-    const double lnZ = log(Z);
-    const double H = lnZ - 0.6931471805599453 * S / Z;
-    const int y = cur_tok != nullptr ? cur_tok[n] : yhat;
-    double u = nan("");                      // a current token outside [0, V) has no probability
-    if (y >= 0 && y < V) {
-      const double xy = (y == yhat) ? static_cast<double>(M) : static_cast<double>(bf16_to_f32(row[y]));
-      u = lnZ - (xy - static_cast<double>(M));
-    }
-    const double din = d_in != nullptr ? static_cast<double>(d_in[n]) : 0.0;
-    const double dout = d_out != nullptr ? static_cast<double>(d_out[n]) : 0.0;
-    const float sc = static_cast<float>(u * (1.0 + din) / (1.0 + dout));
-    maxprob[n] = static_cast<float>(1.0 / Z);
-    entropy[n] = static_cast<float>(H);
-    argmax[n] = yhat;
-    score[n] = sc;
-    s_last = 0;
-    if (topk > 0) {
-      __threadfence();
-      const unsigned seg = static_cast<unsigned>(n / per_seq);
-      const unsigned old = atomicInc(counters + seg, static_cast<unsigned>(per_seq - 1));
-      s_last = (old == static_cast<unsigned>(per_seq - 1));
+    for (int w = 0; w < NW; ++w) {
+      r.Z += red_z[w];
+      r.S += red_s[w];
     }
   }
-  __syncthreads();
-  if (!s_last) return;
+  return r;
+}
 
-  // ---- last CTA of the segment: top-k by (score desc, index asc) ----
+// Thread 0 writes the row's outputs; returns (to thread 0) whether this CTA is
+// the last of its segment to finish.
+__device__ __forceinline__ bool row_write(const RowOut& r, int n, const uint16_t* row, int V, int per_seq,
+                                          const int32_t* cur_tok, const float* d_in, const float* d_out, int topk,
+                                          float* maxprob, float* entropy, int32_t* argmax, float* score,
+                                          uint32_t* counters) {
+  const float Zf = static_cast<float>(r.Z);
+  const float lnZ = logf(Zf);
+  const float H = lnZ - 0.6931471805599453f * static_cast<float>(r.S / r.Z);
+  const int y = cur_tok != nullptr ? cur_tok[n] : r.yhat;
+  float u = __int_as_float(0x7fc00000);   // a current token outside [0, V) has no probability
+  if (y >= 0 && y < V) {
+    const float xy = (y == r.yhat) ? r.M : bf16_to_f32(row[y]);
+    u = lnZ - (xy - r.M);
+  }
+  const float din = d_in != nullptr ? d_in[n] : 0.0f;
+  const float dout = d_out != nullptr ? d_out[n] : 0.0f;
+  maxprob[n] = 1.0f / Zf;
+  entropy[n] = H;
+  argmax[n] = r.yhat;
+  score[n] = u * (1.0f + din) / (1.0f + dout);
+  if (topk <= 0) return false;
   __threadfence();
-  const int seg = n / per_seq;
+  const unsigned seg = static_cast<unsigned>(n / per_seq);
+  const unsigned old = atomicInc(counters + seg, static_cast<unsigned>(per_seq - 1));
+  return old == static_cast<unsigned>(per_seq - 1);
+}
+
+// The last CTA of a segment: top-k by (score desc, index asc) over eligible rows.
+__device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_seq, int sort_n, int topk,
+                                             const float* score, const uint8_t* eligible, int32_t* topk_idx,
+                                             float* topk_score) {
+  __threadfence();
+  const int tid = threadIdx.x, nt = blockDim.x;
   const int base = seg * per_seq;
-  for (int i = tid; i < sort_n; i += kThreads) {
+  for (int i = tid; i < sort_n; i += nt) {
     uint64_t key = 0;
     if (i < per_seq && (eligible == nullptr || eligible[base + i] != 0)) {
       const float sc = __ldcg(score + base + i);
@@ -287,7 +244,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   __syncthreads();
   for (int k = 2; k <= sort_n; k <<= 1) {
     for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = tid; i < sort_n; i += kThreads) {
+      for (int i = tid; i < sort_n; i += nt) {
         const int p = i ^ j;
         if (p > i) {
           const uint64_t x = keys[i], y = keys[p];
@@ -301,7 +258,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       __syncthreads();
     }
   }
-  for (int t = tid; t < topk; t += kThreads) {
+  for (int t = tid; t < topk; t += nt) {
     const uint64_t key = keys[t];
     const bool valid = key != 0;
     topk_idx[static_cast<size_t>(seg) * topk + t] =
@@ -312,16 +269,212 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
 }
 
+// Accumulate U vectors of 8 values; the first index of vector u is i0 + u * istride.
+template <int U>
+__device__ __forceinline__ void acc_batch(RowAcc& a, const uint4 (&w)[U], int i0, int istride) {
+  float x[U][8];
+  float bmax = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    unpack8(w[u], x[u]);
+#pragma unroll
+    for (int k = 0; k < 8; k += 2) bmax = fmax3(bmax, x[u][k], x[u][k + 1]);
+  }
+  if (bmax > a.m) {
+    int idx = 0x7fffffff;
+#pragma unroll
+    for (int u = U - 1; u >= 0; --u)
+#pragma unroll
+      for (int k = 7; k >= 0; --k)
+        if (x[u][k] == bmax) idx = i0 + u * istride + k;
+    raise_max(a, bmax, idx);
+  }
+#pragma unroll
+  for (int u = 0; u < U; ++u) acc_vec8(a, x[u]);
+}
+
+struct ScoreParams {
+  const uint16_t* logits;
+  int V, per_seq;
+  const int32_t* cur_tok;
+  const float* d_in;
+  const float* d_out;
+  const uint8_t* eligible;
+  int topk, sort_n;
+  float* maxprob;
+  float* entropy;
+  int32_t* argmax;
+  float* score;
+  int32_t* topk_idx;
+  float* topk_score;
+  uint32_t* counters;
+};
+
+// ---------------------------------------------------------------------------
+// register-load kernel (any V)
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads, 2) score_kernel(const ScoreParams P) {
+  extern __shared__ uint64_t keys[];
+  __shared__ float red_m[kWarps];
+  __shared__ int red_i[kWarps];
+  __shared__ double red_z[kWarps], red_s[kWarps];
+  __shared__ int s_last;
+
+  const int n = blockIdx.x;
+  const int tid = threadIdx.x;
+  const int V = P.V;
+  const size_t row_off = static_cast<size_t>(n) * V;
+  const uint16_t* row = P.logits + row_off;
+  RowAcc a{-INFINITY, 0x7fffffff, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+
+  // elements before the first 16-byte boundary of the row
+  const int head = min(static_cast<int>((8 - (row_off & 7)) & 7), V);
+  const int nvec = (V - head) / 8;
+  const int tail0 = head + nvec * 8;
+  if (tid < head) acc_scalar(a, bf16_to_f32(row[tid]), tid);
+  const uint4* vrow = reinterpret_cast<const uint4*>(row + head);
+  int v = tid;
+  for (; v + (kUnroll - 1) * kThreads < nvec; v += kUnroll * kThreads) {
+    uint4 w[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) w[u] = ld_stream(vrow + v + u * kThreads);
+    acc_batch<kUnroll>(a, w, head + v * 8, kThreads * 8);
+  }
+  for (; v < nvec; v += kThreads) {
+    uint4 w[1] = {ld_stream(vrow + v)};
+    acc_batch<1>(a, w, head + v * 8, 0);
+  }
+  if (tail0 + tid < V) acc_scalar(a, bf16_to_f32(row[tail0 + tid]), tail0 + tid);
+
+  const RowOut r = row_reduce<kWarps>(a, red_m, red_i, red_z, red_s);
+  if (tid == 0)
+    s_last = row_write(r, n, row, V, P.per_seq, P.cur_tok, P.d_in, P.d_out, P.topk, P.maxprob, P.entropy, P.argmax,
+                       P.score, P.counters);
+  __syncthreads();
+  if (s_last)
+    segment_topk(keys, n / P.per_seq, P.per_seq, P.sort_n, P.topk, P.score, P.eligible, P.topk_idx, P.topk_score);
+}
+
+// ---------------------------------------------------------------------------
+// bulk-copy kernel (rows 16-byte aligned)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void bulk_load(void* smem_dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(smem_dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const ScoreParams P, int* status) {
+  extern __shared__ __align__(128) uint8_t dsmem[];   // ring, reused for top-k keys
+  __shared__ uint64_t bar_full[kRingStages], bar_empty[kRingStages];
+  __shared__ float red_m[kConsumerWarps + 1];
+  __shared__ int red_i[kConsumerWarps + 1];
+  __shared__ double red_z[kConsumerWarps + 1], red_s[kConsumerWarps + 1];
+  __shared__ int s_last, s_abort;
+
+  const int n = blockIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int V = P.V;
+  const uint16_t* row = P.logits + static_cast<size_t>(n) * V;
+  const int nchunks = (V + kChunkElems - 1) / kChunkElems;
+  uint8_t* ring = dsmem;
+
+  if (tid == 0) {
+    for (int s = 0; s < kRingStages; ++s) {
+      mbar_init(&bar_full[s], 1);
+      mbar_init(&bar_empty[s], kConsumerWarps);
+    }
+    s_abort = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  RowAcc a{-INFINITY, 0x7fffffff, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+  if (warp == kConsumerWarps) {
+    // producer: one lane streams the row chunk by chunk
+    if (lane == 0) {
+      for (int c = 0; c < nchunks; ++c) {
+        const int st = c % kRingStages;
+        if (c >= kRingStages && !mbar_wait(&bar_empty[st], ((c / kRingStages) - 1) & 1, &s_abort)) {
+          report_status(status, kStatusTimeout, 200);
+          s_abort = 1;
+          break;
+        }
+        const int elems = min(kChunkElems, V - c * kChunkElems);
+        mbar_arrive_expect_tx(&bar_full[st], static_cast<uint32_t>(elems * 2));
+        bulk_load(ring + st * kChunkBytes, row + static_cast<size_t>(c) * kChunkElems,
+                  static_cast<uint32_t>(elems * 2), &bar_full[st]);
+      }
+      // every copy issued has been consumed once the consumers pass their last
+      // full-barrier wait; nothing is left in flight at the final barrier
+    }
+  } else {
+    for (int c = 0; c < nchunks; ++c) {
+      const int st = c % kRingStages;
+      const bool ok = mbar_wait(&bar_full[st], (c / kRingStages) & 1, &s_abort);
+      if (!__all_sync(0xffffffffu, ok)) {
+        if (lane == 0) {
+          report_status(status, kStatusTimeout, 201);
+          s_abort = 1;
+        }
+        break;
+      }
+      const int elems = min(kChunkElems, V - c * kChunkElems);
+      const uint4* src = reinterpret_cast<const uint4*>(ring + st * kChunkBytes);
+      const int nv = elems / 8;
+      const int v0 = tid, v1 = tid + kConsumerWarps * 32;
+      if (v1 < nv) {
+        uint4 w[2] = {src[v0], src[v1]};
+        acc_batch<2>(a, w, c * kChunkElems + v0 * 8, kConsumerWarps * 32 * 8);
+      } else if (v0 < nv) {
+        uint4 w[1] = {src[v0]};
+        acc_batch<1>(a, w, c * kChunkElems + v0 * 8, 0);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bar_empty[st]);
+    }
+  }
+  // if the producer gave up, wait (bounded) for the copies it already issued
+  if (warp == kConsumerWarps && lane == 0 && s_abort) {
+    for (int c = max(0, nchunks - kRingStages); c < nchunks; ++c)
+      mbar_wait(&bar_full[c % kRingStages], (c / kRingStages) & 1, nullptr, 1000000ull);
+  }
+
+  const RowOut r = row_reduce<kConsumerWarps + 1>(a, red_m, red_i, red_z, red_s);
+  if (tid == 0)
+    s_last = row_write(r, n, row, V, P.per_seq, P.cur_tok, P.d_in, P.d_out, P.topk, P.maxprob, P.entropy, P.argmax,
+                       P.score, P.counters);
+  __syncthreads();
+  if (s_last)
+    segment_topk(reinterpret_cast<uint64_t*>(ring), n / P.per_seq, P.per_seq, P.sort_n, P.topk, P.score,
+                 P.eligible, P.topk_idx, P.topk_score);
+}
+
 }  // namespace
 
-int launch_score(const ScoreArgs& a, int* /*status*/, cudaStream_t stream) {
+int launch_score(const ScoreArgs& a, int* status, cudaStream_t stream) {
   const int per = a.N / a.n_seq;
   int sort_n = 1;
   while (sort_n < per) sort_n <<= 1;
-  const size_t smem = a.topk > 0 ? sizeof(uint64_t) * static_cast<size_t>(sort_n) : 0;
-  score_kernel<<<a.N, kThreads, smem, stream>>>(static_cast<const uint16_t*>(a.logits), a.V, per, a.cur_tok, a.d_in,
-                                                a.d_out, a.eligible, a.topk, sort_n, a.maxprob, a.entropy, a.argmax,
-                                                a.score, a.topk_idx, a.topk_score, a.counters);
+  ScoreParams P{static_cast<const uint16_t*>(a.logits), a.V, per, a.cur_tok, a.d_in, a.d_out, a.eligible,
+                a.topk, sort_n, a.maxprob, a.entropy, a.argmax, a.score, a.topk_idx, a.topk_score, a.counters};
+  const size_t keys_bytes = a.topk > 0 ? sizeof(uint64_t) * static_cast<size_t>(sort_n) : 0;
+  const bool aligned_rows = (a.V % 8) == 0 && (reinterpret_cast<uintptr_t>(a.logits) % 16) == 0;
+  if (aligned_rows) {
+    const size_t smem = std::max(keys_bytes, static_cast<size_t>(kRingStages) * kChunkBytes);
+    static bool attr = false;
+    if (!attr) {
+      if (cudaFuncSetAttribute(score_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(kRingStages * kChunkBytes)) != cudaSuccess)
+        return -3;
+      attr = true;
+    }
+    score_bulk_kernel<<<a.N, kBulkThreads, smem, stream>>>(P, status);
+  } else {
+    score_kernel<<<a.N, kThreads, keys_bytes, stream>>>(P);
+  }
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
 
