@@ -87,19 +87,21 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
 
-// Accumulate 8 consecutive values (one 16-byte vector) whose first index is i0.
-__device__ __forceinline__ void acc_vec8(RowAcc& a, const float (&x)[8]) {
-  float e[8], te[8];
+// 2^t and t 2^t (t = x log2(e) - mref) of the 8 values of one 16-byte vector,
+// on packed pairs; returns the pair sums (lanes: even / odd elements).
+__device__ __forceinline__ void exp_vec8(const uint4& w, uint64_t c2, uint64_t nm2, uint64_t& ez, uint64_t& ets) {
+  const uint32_t v[4] = {w.x, w.y, w.z, w.w};
+  uint64_t e[4], te[4];
 #pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    const float t = fmaf(x[k], kLog2e, -a.mref);
-    e[k] = ex2_approx(t);
-    te[k] = t * e[k];
+  for (int k = 0; k < 4; ++k) {
+    const uint64_t t2 = f2_fma(f2_pack(__uint_as_float(v[k] << 16), __uint_as_float(v[k] & 0xffff0000u)), c2, nm2);
+    float t0, t1;
+    f2_unpack(t2, t0, t1);
+    e[k] = f2_pack(ex2_approx(t0), ex2_approx(t1));
+    te[k] = f2_mul(t2, e[k]);
   }
-  const float pz = ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
-  const float ps = ((te[0] + te[1]) + (te[2] + te[3])) + ((te[4] + te[5]) + (te[6] + te[7]));
-  kahan_add(a.z, a.zc, pz);
-  kahan_add(a.s, a.sc, ps);
+  ez = f2_add(f2_add(e[0], e[1]), f2_add(e[2], e[3]));
+  ets = f2_add(f2_add(te[0], te[1]), f2_add(te[2], te[3]));
 }
 
 __device__ __forceinline__ void acc_scalar(RowAcc& a, float x, int idx) {
@@ -272,25 +274,42 @@ __device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_se
 // Accumulate U vectors of 8 values; the first index of vector u is i0 + u * istride.
 template <int U>
 __device__ __forceinline__ void acc_batch(RowAcc& a, const uint4 (&w)[U], int i0, int istride) {
-  float x[U][8];
   float bmax = -INFINITY;
 #pragma unroll
   for (int u = 0; u < U; ++u) {
-    unpack8(w[u], x[u]);
+    const uint32_t v[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
 #pragma unroll
-    for (int k = 0; k < 8; k += 2) bmax = fmax3(bmax, x[u][k], x[u][k + 1]);
+    for (int k = 0; k < 4; ++k)
+      bmax = fmax3(bmax, __uint_as_float(v[k] << 16), __uint_as_float(v[k] & 0xffff0000u));
   }
   if (bmax > a.m) {
     int idx = 0x7fffffff;
 #pragma unroll
-    for (int u = U - 1; u >= 0; --u)
+    for (int u = U - 1; u >= 0; --u) {
+      float x[8];
+      unpack8(w[u], x);
 #pragma unroll
       for (int k = 7; k >= 0; --k)
-        if (x[u][k] == bmax) idx = i0 + u * istride + k;
+        if (x[k] == bmax) idx = i0 + u * istride + k;
+    }
     raise_max(a, bmax, idx);
   }
+  const uint64_t c2 = f2_pack(kLog2e, kLog2e);
+  const uint64_t nm2 = f2_pack(-a.mref, -a.mref);
+  uint64_t ez, ets;
+  exp_vec8(w[0], c2, nm2, ez, ets);
 #pragma unroll
-  for (int u = 0; u < U; ++u) acc_vec8(a, x[u]);
+  for (int u = 1; u < U; ++u) {
+    uint64_t ez2, ets2;
+    exp_vec8(w[u], c2, nm2, ez2, ets2);
+    ez = f2_add(ez, ez2);
+    ets = f2_add(ets, ets2);
+  }
+  float z0, z1, s0, s1;
+  f2_unpack(ez, z0, z1);
+  f2_unpack(ets, s0, s1);
+  kahan_add(a.z, a.zc, z0 + z1);
+  kahan_add(a.s, a.sc, s0 + s1);
 }
 
 struct ScoreParams {
