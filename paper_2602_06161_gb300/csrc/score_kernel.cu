@@ -18,9 +18,9 @@
 //
 // Two ways to stream a row:
 //  * score_bulk_kernel (rows 16-byte aligned, V % 8 == 0): a producer warp
-//    issues cp.async.bulk copies of 8 KB chunks into a 6-stage shared-memory
+//    issues cp.async.bulk copies of 16 KB chunks into a 4-stage shared-memory
 //    ring (mbarrier full / empty), 8 consumer warps reduce from shared memory;
-//    bytes in flight do not cost registers, and 4 CTAs share an SM.
+//    bytes in flight do not cost registers, and 3 CTAs share an SM.
 //  * score_kernel (any V): 16-byte non-allocating global loads, scalar head and
 //    tail for rows that do not start on a 16-byte boundary.
 #include <math.h>
@@ -39,9 +39,10 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kUnroll = 4;
 constexpr int kConsumerWarps = 8;          // bulk kernel: consumers + 1 producer warp
 constexpr int kBulkThreads = (kConsumerWarps + 1) * 32;
-constexpr int kChunkElems = 4096;          // 8 KB of bf16 per bulk copy
+constexpr int kChunkElems = 8192;          // 16 KB of bf16 per bulk copy
 constexpr int kChunkBytes = kChunkElems * 2;
-constexpr int kRingStages = 6;
+constexpr int kRingStages = 4;
+constexpr int kVecPerThread = kChunkElems / 8 / (kConsumerWarps * 32);   // 4
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct RowAcc {
@@ -86,23 +87,6 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
 }
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
-
-// 2^t and t 2^t (t = x log2(e) - mref) of the 8 values of one 16-byte vector,
-// on packed pairs; returns the pair sums (lanes: even / odd elements).
-__device__ __forceinline__ void exp_vec8(const uint4& w, uint64_t c2, uint64_t nm2, uint64_t& ez, uint64_t& ets) {
-  const uint32_t v[4] = {w.x, w.y, w.z, w.w};
-  uint64_t e[4], te[4];
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const uint64_t t2 = f2_fma(f2_pack(__uint_as_float(v[k] << 16), __uint_as_float(v[k] & 0xffff0000u)), c2, nm2);
-    float t0, t1;
-    f2_unpack(t2, t0, t1);
-    e[k] = f2_pack(ex2_approx(t0), ex2_approx(t1));
-    te[k] = f2_mul(t2, e[k]);
-  }
-  ez = f2_add(f2_add(e[0], e[1]), f2_add(e[2], e[3]));
-  ets = f2_add(f2_add(te[0], te[1]), f2_add(te[2], te[3]));
-}
 
 __device__ __forceinline__ void acc_scalar(RowAcc& a, float x, int idx) {
   if (x > a.m) raise_max(a, x, idx);
@@ -272,42 +256,45 @@ __device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_se
 }
 
 // Accumulate U vectors of 8 values; the first index of vector u is i0 + u * istride.
+// Per pair of values: one packed FMA for t, two ex2, one packed add into Z and
+// one packed FMA into S; two independent accumulator chains.
 template <int U>
 __device__ __forceinline__ void acc_batch(RowAcc& a, const uint4 (&w)[U], int i0, int istride) {
+  float x[U][8];
   float bmax = -INFINITY;
 #pragma unroll
   for (int u = 0; u < U; ++u) {
-    const uint32_t v[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+    unpack8(w[u], x[u]);
 #pragma unroll
-    for (int k = 0; k < 4; ++k)
-      bmax = fmax3(bmax, __uint_as_float(v[k] << 16), __uint_as_float(v[k] & 0xffff0000u));
+    for (int k = 0; k < 8; k += 2) bmax = fmax3(bmax, x[u][k], x[u][k + 1]);
   }
   if (bmax > a.m) {
     int idx = 0x7fffffff;
 #pragma unroll
-    for (int u = U - 1; u >= 0; --u) {
-      float x[8];
-      unpack8(w[u], x);
+    for (int u = U - 1; u >= 0; --u)
 #pragma unroll
       for (int k = 7; k >= 0; --k)
-        if (x[k] == bmax) idx = i0 + u * istride + k;
-    }
+        if (x[u][k] == bmax) idx = i0 + u * istride + k;
     raise_max(a, bmax, idx);
   }
   const uint64_t c2 = f2_pack(kLog2e, kLog2e);
   const uint64_t nm2 = f2_pack(-a.mref, -a.mref);
-  uint64_t ez, ets;
-  exp_vec8(w[0], c2, nm2, ez, ets);
+  uint64_t z[2] = {0, 0}, sacc[2] = {0, 0};
 #pragma unroll
-  for (int u = 1; u < U; ++u) {
-    uint64_t ez2, ets2;
-    exp_vec8(w[u], c2, nm2, ez2, ets2);
-    ez = f2_add(ez, ez2);
-    ets = f2_add(ets, ets2);
+  for (int u = 0; u < U; ++u) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint64_t t2 = f2_fma(f2_pack(x[u][2 * k], x[u][2 * k + 1]), c2, nm2);
+      float t0, t1;
+      f2_unpack(t2, t0, t1);
+      const uint64_t e2 = f2_pack(ex2_approx(t0), ex2_approx(t1));
+      z[k & 1] = f2_add(z[k & 1], e2);
+      sacc[k & 1] = f2_fma(t2, e2, sacc[k & 1]);
+    }
   }
   float z0, z1, s0, s1;
-  f2_unpack(ez, z0, z1);
-  f2_unpack(ets, s0, s1);
+  f2_unpack(f2_add(z[0], z[1]), z0, z1);
+  f2_unpack(f2_add(sacc[0], sacc[1]), s0, s1);
   kahan_add(a.z, a.zc, z0 + z1);
   kahan_add(a.s, a.sc, s0 + s1);
 }
@@ -385,7 +372,7 @@ __device__ __forceinline__ void bulk_load(void* smem_dst, const void* src, uint3
       : "memory");
 }
 
-__global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const ScoreParams P, int* status) {
+__global__ void __launch_bounds__(kBulkThreads, 3) score_bulk_kernel(const ScoreParams P, int* status) {
   extern __shared__ __align__(128) uint8_t dsmem[];   // ring, reused for top-k keys
   __shared__ uint64_t bar_full[kRingStages], bar_empty[kRingStages];
   __shared__ float red_m[kConsumerWarps + 1];
@@ -443,13 +430,17 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
       const int elems = min(kChunkElems, V - c * kChunkElems);
       const uint4* src = reinterpret_cast<const uint4*>(ring + st * kChunkBytes);
       const int nv = elems / 8;
-      const int v0 = tid, v1 = tid + kConsumerWarps * 32;
-      if (v1 < nv) {
-        uint4 w[2] = {src[v0], src[v1]};
-        acc_batch<2>(a, w, c * kChunkElems + v0 * 8, kConsumerWarps * 32 * 8);
-      } else if (v0 < nv) {
-        uint4 w[1] = {src[v0]};
-        acc_batch<1>(a, w, c * kChunkElems + v0 * 8, 0);
+      constexpr int kStride = kConsumerWarps * 32;
+      if (tid + (kVecPerThread - 1) * kStride < nv) {
+        uint4 w[kVecPerThread];
+#pragma unroll
+        for (int u = 0; u < kVecPerThread; ++u) w[u] = src[tid + u * kStride];
+        acc_batch<kVecPerThread>(a, w, c * kChunkElems + tid * 8, kStride * 8);
+      } else {
+        for (int v = tid; v < nv; v += kStride) {
+          uint4 w[1] = {src[v]};
+          acc_batch<1>(a, w, c * kChunkElems + v * 8, 0);
+        }
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&bar_empty[st]);
