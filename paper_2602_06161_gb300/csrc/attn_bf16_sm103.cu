@@ -17,6 +17,11 @@
 //   warps 4-7  softmax + epilogue of Q tile 1
 //   warp  8    tensor-memory allocation; lane 0 issues tcgen05.mma
 //   warp  9    lane 0 issues TMA loads (Q once, K/V through a 2-stage ring)
+//   warps 10-11 complete the producer warpgroup (register donors, no work)
+// Registers: launched at 168 per thread (12 warps); the producer warpgroup
+// gives back down to 136 and the two softmax warpgroups take 184 each
+// (setmaxnreg), so the 128-column softmax rows stay in registers without
+// spilling.
 // Tensor memory (512 columns): S0 | S1 | O0 | O1, 128 fp32 columns each; the
 // bf16 probabilities P of tile t overwrite the first 64 columns of S_t and
 // feed the P.V product straight from tensor memory.
@@ -43,7 +48,11 @@ constexpr int kRowsPerCta = kNQ * kBM;
 constexpr int kStages = 2;
 constexpr int kTileBytes = kBM * kD * 2;  // 32 KB
 constexpr int kBoxBytes = kTileBytes / 2; // one 64-column, 128-byte-swizzled box
-constexpr int kThreads = 320;
+constexpr int kThreads = 384;
+constexpr int kLaunchRegs = 168;          // registers per thread at launch (65536 / 384, rounded to 8)
+constexpr int kSoftmaxRegs = 184;         // 2 * 128 * 184 + 128 * 136 == 384 * 168
+constexpr int kProducerRegs = 136;
+static_assert(2 * 128 * kSoftmaxRegs + 128 * kProducerRegs <= kThreads * kLaunchRegs, "register split");
 constexpr int kMmaWarp = 8;
 constexpr int kTmaWarp = 9;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
@@ -128,7 +137,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   const uint32_t tbase = sm.tmem_base;
 
-  if (warp == kTmaWarp) {
+  if (warp >= kMmaWarp) {
+   setmaxnreg_dec<kProducerRegs>();
+   if (warp == kTmaWarp) {
     // ---------------- TMA producer ----------------
     if (lane == 0) {
       tma_prefetch_desc(&tm_q);
@@ -227,7 +238,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       umma_commit(&sm.bar_drain);
       mbar_wait(&sm.bar_drain, 0, nullptr);
     }
+   }
   } else {
+    setmaxnreg_inc<kSoftmaxRegs>();
     // ---------------- softmax (warps 0-7) ----------------
     const int qt = warp >> 2;
     const int r = tid & (kBM - 1);
@@ -422,6 +435,10 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
     if (cudaFuncSetAttribute(attn_bf16_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
         cudaSuccess)
       return -3;
+    // the register split inside the kernel assumes exactly kLaunchRegs per thread at launch;
+    // any other count could leave setmaxnreg.inc waiting, so refuse to launch
+    cudaFuncAttributes fa;
+    if (cudaFuncGetAttributes(&fa, attn_bf16_kernel) != cudaSuccess || fa.numRegs != kLaunchRegs) return -2;
     attr_set = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
