@@ -139,6 +139,35 @@ int cover_score_fwd(const void* logits, int N, int V, int n_seq,
                     void* workspace, void* stream);
 
 /*
+ * cover_score_fwd without a workspace argument. The paper has no counterpart:
+ * this entry point exists for callers that cannot allocate device memory for
+ * a workspace - for example a serving loop that reserves all of its GPU
+ * memory up front and forbids allocation afterwards, or a plugin interface
+ * that hands the library its inputs and outputs but no allocator.
+ *
+ * Same arguments, layouts, results and errors as cover_score_fwd. The
+ * per-sequence counters that cover_score_fwd keeps in the caller's workspace
+ * live here in one fixed device array of the library, sized for at most
+ * COVER_NOALLOC_MAX_SEQ (4096) sequences; n_seq beyond that returns
+ * COVER_ERR_INVALID_ARG. Every device that loads the library holds this
+ * 16 KB array until the process exits. The call allocates nothing: no
+ * cudaMalloc / cudaFree, no allocating library routine; it clears the
+ * counters it uses with an asynchronous memset on `stream`, then launches.
+ *
+ * The first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current); make that first call
+ * before any stream capture begins. All calls share the one array: calls
+ * that overlap on the GPU (different streams, or different host threads
+ * without ordering) race on it and can return wrong top-k results.
+ */
+#define COVER_NOALLOC_MAX_SEQ 4096
+int cover_score_fwd_noalloc(const void* logits, int N, int V, int n_seq,
+                            const int32_t* cur_tok, const float* d_in, const float* d_out,
+                            const uint8_t* eligible, int topk,
+                            float* maxprob, float* entropy, int32_t* argmax, float* score,
+                            int32_t* topk_idx, float* topk_score, void* stream);
+
+/*
  * Synchronises `stream`, then returns and clears the current device's status
  * word: COVER_OK, or COVER_ERR_DEVICE_TIMEOUT if a kernel gave up on a
  * bounded wait since the last call. Returns COVER_ERR_CUDA if the

@@ -4,7 +4,8 @@ The compute path is libcover.so (hand-written CUDA, C ABI in include/cover.h);
 this package only loads it and marshals torch tensors into it.
 """
 from .api import (  # noqa: F401
-    cover_attn_fwd, cover_attn_fwd_f32, cover_seed_route, cover_score_fwd, cover_score_workspace_bytes,
+    cover_attn_fwd, cover_attn_fwd_f32, cover_seed_route, cover_score_fwd, cover_score_fwd_noalloc,
+    cover_score_workspace_bytes,
     score_workspace, cover_device_status, cover_status_str, cover_debug_umma_tile, cover_debug_wait_timeout,
 )
 from ._lib import CoverError, load as load_library  # noqa: F401

@@ -152,6 +152,40 @@ def cover_score_fwd(logits, n_seq: int, topk: int, *, cur_tok=None, d_in=None, d
     return out
 
 
+def cover_score_fwd_noalloc(logits, n_seq: int, topk: int, *, cur_tok=None, d_in=None, d_out=None, eligible=None,
+                            out=None, stream=None):
+    """cover_score_fwd without a workspace: for callers that cannot allocate device memory.
+
+    The per-sequence counters live in a fixed device array of the library
+    (at most 4096 sequences). Calls that overlap on the GPU race on that array.
+    The first call on a device looks up the array's address; make it before
+    any stream capture. Returns the same dict as cover_score_fwd.
+    """
+    _need(logits, "logits", torch.bfloat16, 2)
+    N, V = logits.shape
+    dev = logits.device
+    for name, t, dt in (("cur_tok", cur_tok, torch.int32), ("d_in", d_in, torch.float32),
+                        ("d_out", d_out, torch.float32), ("eligible", eligible, torch.uint8)):
+        if t is not None:
+            _need(t, name, dt, 1)
+    if out is None:
+        out = dict(
+            maxprob=torch.empty(N, dtype=torch.float32, device=dev),
+            entropy=torch.empty(N, dtype=torch.float32, device=dev),
+            argmax=torch.empty(N, dtype=torch.int32, device=dev),
+            score=torch.empty(N, dtype=torch.float32, device=dev),
+            topk_idx=torch.empty((n_seq, max(topk, 0)), dtype=torch.int32, device=dev),
+            topk_score=torch.empty((n_seq, max(topk, 0)), dtype=torch.float32, device=dev),
+        )
+    code = _lib.load().cover_score_fwd_noalloc(
+        _ptr(logits), N, V, n_seq, _ptr(cur_tok), _ptr(d_in), _ptr(d_out), _ptr(eligible), topk,
+        _ptr(out["maxprob"]), _ptr(out["entropy"]), _ptr(out["argmax"]), _ptr(out["score"]),
+        _ptr(out["topk_idx"]) if topk > 0 else None, _ptr(out["topk_score"]) if topk > 0 else None,
+        _stream(stream))
+    _lib.check("cover_score_fwd_noalloc", code)
+    return out
+
+
 def cover_device_status(stream=None) -> int:
     """Synchronise the stream; return and clear the device status word (0 = OK)."""
     return int(_lib.load().cover_device_status(_stream(stream)))

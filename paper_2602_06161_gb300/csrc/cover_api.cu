@@ -113,6 +113,27 @@ int cover_score_fwd(const void* logits, int N, int V, int n_seq, const int32_t* 
   return cover::launch_score(a, st, static_cast<cudaStream_t>(stream));
 }
 
+int cover_score_fwd_noalloc(const void* logits, int N, int V, int n_seq, const int32_t* cur_tok, const float* d_in,
+                            const float* d_out, const uint8_t* eligible, int topk, float* maxprob, float* entropy,
+                            int32_t* argmax, float* score, int32_t* topk_idx, float* topk_score, void* stream) {
+  if (logits == nullptr || maxprob == nullptr || entropy == nullptr || argmax == nullptr || score == nullptr)
+    return COVER_ERR_INVALID_ARG;
+  if (N < 1 || V < 1 || n_seq < 1 || N % n_seq != 0) return COVER_ERR_INVALID_ARG;
+  if (n_seq > cover::kNoAllocMaxSegments) return COVER_ERR_INVALID_ARG;
+  const int per = N / n_seq;
+  if (per > 4096) return COVER_ERR_INVALID_ARG;
+  if (topk < 0 || topk > per) return COVER_ERR_INVALID_ARG;
+  if (topk > 0 && topk_idx == nullptr) return COVER_ERR_INVALID_ARG;
+  if (!aligned(logits, 16) || !aligned(maxprob, 4) || !aligned(entropy, 4) || !aligned(argmax, 4) ||
+      !aligned(score, 4))
+    return COVER_ERR_INVALID_ARG;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  cover::ScoreArgs a{logits, N, V, n_seq, cur_tok, d_in, d_out, eligible, topk, maxprob, entropy, argmax,
+                     score, topk_idx, topk_score, nullptr};
+  return cover::launch_score_noalloc(a, st, static_cast<cudaStream_t>(stream));
+}
+
 int cover_device_status(void* stream) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int* st = status_block();

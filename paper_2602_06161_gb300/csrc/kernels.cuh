@@ -46,6 +46,11 @@ struct ScoreArgs {
 
 int launch_score(const ScoreArgs& a, int* status, cudaStream_t stream);
 
+// Same as launch_score, with the counters in a fixed device array of the
+// library (a.counters is ignored). Returns -1 if a.n_seq > kNoAllocMaxSegments.
+constexpr int kNoAllocMaxSegments = 4096;
+int launch_score_noalloc(ScoreArgs a, int* status, cudaStream_t stream);
+
 int launch_umma_tile(const void* a, const void* b, const void* p, const void* v, float* c1, float* c2, int* status,
                      cudaStream_t stream);
 int launch_wait_timeout(uint64_t limit_ns, int* status, cudaStream_t stream);

@@ -27,6 +27,7 @@
 #include <stdint.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "kernels.cuh"
 #include "ptx.cuh"
@@ -486,6 +487,50 @@ int launch_score(const ScoreArgs& a, int* status, cudaStream_t stream) {
     score_kernel<<<a.N, kThreads, keys_bytes, stream>>>(P);
   }
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant: the same kernels, with the per-segment counters in
+// a fixed device array of this library instead of a caller workspace.
+// ---------------------------------------------------------------------------
+namespace {
+
+// Counters for at most kNoAllocMaxSegments segments (16 KB). Every device that
+// loads the library holds one copy until the process exits.
+static __device__ __align__(256) uint32_t g_noalloc_counters[kNoAllocMaxSegments];
+
+constexpr int kMaxDevicesNoAlloc = 64;
+uint32_t* g_noalloc_addr[kMaxDevicesNoAlloc];
+std::mutex g_noalloc_mu;
+
+// Device address of the counter array on the current device. In host code the
+// array's name is only a host-side stand-in, so the address is looked up once
+// per device (with that device current) and cached.
+uint32_t* noalloc_counters() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevicesNoAlloc) return nullptr;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (g_noalloc_addr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_counters) != cudaSuccess || p == nullptr) return nullptr;
+    g_noalloc_addr[dev] = static_cast<uint32_t*>(p);
+  }
+  return g_noalloc_addr[dev];
+}
+
+}  // namespace
+
+int launch_score_noalloc(ScoreArgs a, int* status, cudaStream_t stream) {
+  if (a.n_seq > kNoAllocMaxSegments) return -1;
+  uint32_t* counters = noalloc_counters();
+  if (counters == nullptr) return -3;
+  // the array keeps whatever the previous call left: the counters this call
+  // uses must start at zero
+  if (a.topk > 0 &&
+      cudaMemsetAsync(counters, 0, sizeof(uint32_t) * static_cast<size_t>(a.n_seq), stream) != cudaSuccess)
+    return -3;
+  a.counters = counters;
+  return launch_score(a, status, stream);
 }
 
 }  // namespace cover
