@@ -409,8 +409,10 @@ def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, iters=2
 # the oracle on the host cores (cpu_baseline and the reference arm)
 # ----------------------------------------------------------------------------
 
-SAMPLE_HEADS = 8          # of the 256 (b, hq) heads of the workload
-SAMPLE_SCORE_ROWS = 64    # of the 2048 scored rows (same 1/32 fraction)
+SAMPLE_HEADS = 128        # of the 256 (b, hq) heads of the workload (all host threads)
+SAMPLE_SCORE_ROWS = 1024  # of the 2048 scored rows (the same fraction, 1/2)
+SAMPLE_HEADS_1T = 16      # single-thread run: 1/16 of the heads and rows
+SAMPLE_SCORE_ROWS_1T = 128
 
 
 def oracle_sample_step(ai, si, wl, heads, rows):
@@ -452,9 +454,9 @@ def cpu_baseline():
     for threads in (n, 1):
         env = dict(os.environ, OMP_NUM_THREADS=str(threads), OPENBLAS_NUM_THREADS=str(threads),
                    MKL_NUM_THREADS=str(threads), CUDA_VISIBLE_DEVICES="")
+        heads, rows = (SAMPLE_HEADS, SAMPLE_SCORE_ROWS) if threads == n else (SAMPLE_HEADS_1T, SAMPLE_SCORE_ROWS_1T)
         code = ("import json,sys; sys.path.insert(0, %r); import bench; "
-                "fl, t = bench._cpu_worker(%d, %d, 1); print(json.dumps([fl, t]))" %
-                (ROOT, SAMPLE_HEADS, SAMPLE_SCORE_ROWS))
+                "fl, t = bench._cpu_worker(%d, %d, 1); print(json.dumps([fl, t]))" % (ROOT, heads, rows))
         r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, cwd=ROOT,
                            timeout=900)
         if r.returncode != 0:
@@ -469,7 +471,8 @@ def cpu_baseline():
     out = {"value": round(fl / t / 1e12, 6), "unit": UNIT, "cores": n, "kind": "oracle",
            "sample": f"{SAMPLE_HEADS} of {256} attention heads (full L=2048, all their seed rows through "
                      f"explicit leave-one-out views) + {SAMPLE_SCORE_ROWS} of 2048 scored rows; "
-                     f"fp64 numpy, {t:.1f} s"}
+                     f"fp64 numpy, {t:.1f} s on {n} threads; value_1_thread from "
+                     f"{SAMPLE_HEADS_1T} heads + {SAMPLE_SCORE_ROWS_1T} rows"}
     if res.get(1) is not None:
         out["value_1_thread"] = round(res[1][0] / res[1][1] / 1e12, 6)
     return out
