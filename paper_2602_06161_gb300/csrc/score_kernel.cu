@@ -8,8 +8,9 @@
 // with p = softmax(logits) at temperature 1. Each thread keeps, for its share
 // of the row, the running maximum m (exact bf16 compare, first index kept),
 // Z = sum 2^t and S = sum t 2^t with t = x log2(e) - m log2(e), Kahan
-// compensated; partials are re-referenced to the row maximum and summed in
-// fp64. Then c = 1/Z, H = ln Z - ln(2) S / Z, u = ln Z - (x_y - m).
+// compensated; partials are re-referenced to the row maximum, summed across
+// each warp in fp32 with error-free TwoSum pairs and across warps in fp64.
+// Then c = 1/Z, H = ln Z - ln(2) S / Z, u = ln Z - (x_y - m).
 //
 // Top-k (Section 5.3): the last CTA to finish a segment (sequence) - found
 // with a self-resetting atomicInc counter per segment - sorts the segment's
@@ -18,9 +19,9 @@
 //
 // Two ways to stream a row:
 //  * score_bulk_kernel (rows 16-byte aligned, V % 8 == 0): a producer warp
-//    issues cp.async.bulk copies of 16 KB chunks into a 4-stage shared-memory
+//    issues cp.async.bulk copies of 16 KB chunks into a 3-stage shared-memory
 //    ring (mbarrier full / empty), 8 consumer warps reduce from shared memory;
-//    bytes in flight do not cost registers, and 3 CTAs share an SM.
+//    bytes in flight do not cost registers, and 4 CTAs share an SM.
 //  * score_kernel (any V): 16-byte non-allocating global loads, scalar head and
 //    tail for rows that do not start on a 16-byte boundary.
 #include <math.h>
@@ -42,7 +43,7 @@ constexpr int kConsumerWarps = 8;          // bulk kernel: consumers + 1 produce
 constexpr int kBulkThreads = (kConsumerWarps + 1) * 32;
 constexpr int kChunkElems = 8192;          // 16 KB of bf16 per bulk copy
 constexpr int kChunkBytes = kChunkElems * 2;
-constexpr int kRingStages = 4;
+constexpr int kRingStages = 3;
 constexpr int kVecPerThread = kChunkElems / 8 / (kConsumerWarps * 32);   // 4
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -156,23 +157,33 @@ __device__ __forceinline__ RowOut row_reduce(const RowAcc& a, float* red_m, int*
     }
   }
   const float Mref = M * kLog2e;
-  double zd = 0.0, sd = 0.0;
+  // partials re-referenced to the row maximum, summed across the warp in fp32
+  // with error-free TwoSum pairs (value, rounding error); fp64 only for the
+  // final sum of the per-warp results
+  float z = 0.0f, ze = 0.0f, sv = 0.0f, se = 0.0f;
   if (a.m != -INFINITY) {
     const float d = a.mref - Mref;
     const float f = ex2_approx(d);
-    const float z = a.z - a.zc;
-    const float s = a.s - a.sc;
-    zd = static_cast<double>(f * z);
-    sd = static_cast<double>(f * fmaf(d, z, s));
+    const float zz = a.z - a.zc;
+    const float ss = a.s - a.sc;
+    z = f * zz;
+    sv = f * fmaf(d, zz, ss);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    zd += __shfl_xor_sync(0xffffffffu, zd, o);
-    sd += __shfl_xor_sync(0xffffffffu, sd, o);
+    const float z2 = __shfl_xor_sync(0xffffffffu, z, o), ze2 = __shfl_xor_sync(0xffffffffu, ze, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, sv, o), se2 = __shfl_xor_sync(0xffffffffu, se, o);
+    float t = z + z2, bb = t - z;
+    ze += ze2 + ((z - (t - bb)) + (z2 - bb));
+    z = t;
+    t = sv + s2;
+    bb = t - sv;
+    se += se2 + ((sv - (t - bb)) + (s2 - bb));
+    sv = t;
   }
   if (lane == 0) {
-    red_z[warp] = zd;
-    red_s[warp] = sd;
+    red_z[warp] = static_cast<double>(z) + static_cast<double>(ze);
+    red_s[warp] = static_cast<double>(sv) + static_cast<double>(se);
   }
   __syncthreads();
   RowOut r{M, I, 0.0, 0.0};
@@ -373,7 +384,7 @@ __device__ __forceinline__ void bulk_load(void* smem_dst, const void* src, uint3
       : "memory");
 }
 
-__global__ void __launch_bounds__(kBulkThreads, 3) score_bulk_kernel(const ScoreParams P, int* status) {
+__global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const ScoreParams P, int* status) {
   extern __shared__ __align__(128) uint8_t dsmem[];   // ring, reused for top-k keys
   __shared__ uint64_t bar_full[kRingStages], bar_empty[kRingStages];
   __shared__ float red_m[kConsumerWarps + 1];
