@@ -342,24 +342,32 @@ def run_ours(args):
         "clocks": clocks.summary(),
     }
 
-    # ---------------- secondary: seed overhead and long context ----------------
+    # ---------------- secondary: every named workload ----------------
     if not args.no_secondary:
-        ov4 = seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops)
+        per = {WORKLOAD: seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops)}
         del q, kc, vc, km, vm, logits
         torch.cuda.empty_cache()
-        lw = W.WORKLOADS[LONG_WORKLOAD]
-        li = lw.attn_inputs()
-        lq, lkc, lvc = bf16_dev(li.q, torch), bf16_dev(li.k_cached, torch), bf16_dev(li.v_cached, torch)
-        lkm, lvm = bf16_dev(li.k_seedmask, torch), bf16_dev(li.v_seedmask, torch)
-        lseeds = torch.from_numpy(li.seed_idx).cuda()
-        lout = torch.empty_like(lq)
-        llse = torch.empty((lw.B, lw.Hq, lw.L), dtype=torch.float32, device="cuda")
-        ov5 = seed_overhead(api, torch, lq, lkc, lvc, lkm, lvm, lseeds, lout, llse, lw.attn_flops)
-        result["overhead_vs_no_seed"] = {WORKLOAD: ov4["overhead"], LONG_WORKLOAD: ov5["overhead"]}
-        result["seed_timing"] = {WORKLOAD: ov4, LONG_WORKLOAD: ov5}
-        result["long_context"] = {"workload": LONG_WORKLOAD, "tflops": ov5["tflops_seeded"],
-                                  "frac_of_peak": round(ov5["tflops_seeded"] / peak, 4),
+        scoring_all = {WORKLOAD: scoring["gbs"]}
+        for name in ("llada_mha_l512", "dream_gqa_l1024", LONG_WORKLOAD):
+            ow = W.WORKLOADS[name]
+            oi = ow.attn_inputs()
+            oq, okc, ovc = bf16_dev(oi.q, torch), bf16_dev(oi.k_cached, torch), bf16_dev(oi.v_cached, torch)
+            okm, ovm = bf16_dev(oi.k_seedmask, torch), bf16_dev(oi.v_seedmask, torch)
+            oseeds = torch.from_numpy(oi.seed_idx).cuda()
+            oout = torch.empty_like(oq)
+            olse = torch.empty((ow.B, ow.Hq, ow.L), dtype=torch.float32, device="cuda")
+            per[name] = seed_overhead(api, torch, oq, okc, ovc, okm, ovm, oseeds, oout, olse, ow.attn_flops)
+            del oq, okc, ovc, okm, ovm, oseeds, oout, olse
+            osi = ow.score_inputs()
+            if osi is not None:
+                scoring_all[name] = score_gbs(api, torch, osi)
+            torch.cuda.empty_cache()
+        result["overhead_vs_no_seed"] = {k2: v2["overhead"] for k2, v2 in per.items()}
+        result["seed_timing"] = per
+        result["long_context"] = {"workload": LONG_WORKLOAD, "tflops": per[LONG_WORKLOAD]["tflops_seeded"],
+                                  "frac_of_peak": round(per[LONG_WORKLOAD]["tflops_seeded"] / peak, 4),
                                   "peak_source": roofline["peak_source"]}
+        result["scoring_gbs"] = scoring_all
         status = api.cover_device_status()
         if status != 0:
             raise RuntimeError(f"device status {api.cover_status_str(status)} in the secondary runs")
@@ -370,6 +378,24 @@ def run_ours(args):
         import torch.distributed as dist
         dist.destroy_process_group()
     return result if rank == 0 else None
+
+
+def score_gbs(api, torch, si, iters=20):
+    """Median scoring time on one workload's logits (cold L2: the logits exceed it); GB/s of algorithmic bytes."""
+    logits = bf16_dev(si.logits, torch)
+    wsp = api.score_workspace(si.n_seq)
+    out = api.cover_score_fwd(logits, si.n_seq, si.topk, workspace=wsp)
+    stream = torch.cuda.current_stream()
+    ts = []
+    for _ in range(iters):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        api.cover_score_fwd(logits, si.n_seq, si.topk, workspace=wsp, out=out)
+        b.record(stream)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    nbytes = si.N * si.V * 2 + si.N * 20 + si.n_seq * si.topk * 8
+    return round(nbytes / (statistics.median(ts) * 1e-3) / 1e9, 1)
 
 
 def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, iters=20):
