@@ -192,33 +192,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t dq0 = sdesc_sw128(smem_u32(sm.q[0]), 16, 1024);
       const uint64_t dk0 = sdesc_sw128(smem_u32(sm.k[0]), 16, 1024);
       const uint64_t dv0 = sdesc_sw128(smem_u32(sm.v[0]), kBoxBytes, 1024);
+      // Per KV tile j: PV(0, j-1), S(0, j), PV(1, j-1), S(1, j). Each wait sits right after a
+      // group of products has been queued, so the tensor pipe works while the thread waits.
       for (int j = 0; j <= nkv && ok; ++j) {
-        const int st = j & 1;
-        if (j < nkv) {
-          ok = mbar_wait(&sm.bar_k_full[st], (j >> 1) & 1, &sm.abort);
-          if (!ok) break;
-        }
-        if (j > 0) {
-          const int pst = (j - 1) & 1;
-          ok = mbar_wait(&sm.bar_v_full[pst], ((j - 1) >> 1) & 1, &sm.abort);
-          if (!ok) break;
-        }
-        tc_fence_after_sync();
-        for (int t = 0; t < kNQ && ok; ++t) {
+        const int st = j & 1, pst = (j - 1) & 1;
+        for (int t = 0; t < kNQ; ++t) {
           if (j > 0) {
-            // O_t += P_t(j-1) . V(j-1); P from tensor memory, V MN-major from shared memory
             ok = mbar_wait(&sm.bar_p_full[t], (j - 1) & 1, &sm.abort);
             if (!ok) break;
             tc_fence_after_sync();
-            const int pst = (j - 1) & 1;
+            // O_t += P_t(j-1) . V(j-1); P from tensor memory, V MN-major from shared memory
 #pragma unroll
             for (int ks = 0; ks < kBN / 16; ++ks)
               umma_ts(tbase + col_o(t), tbase + col_s(t) + 8 * ks,
-                      dv0 + pst * kTileDesc + static_cast<uint64_t>((ks * 2048) >> 4),
-                      id_pv, (j > 1 || ks > 0) ? 1u : 0u);
+                      dv0 + pst * kTileDesc + static_cast<uint64_t>((ks * 2048) >> 4), id_pv,
+                      (j > 1 || ks > 0) ? 1u : 0u);
             if (j == nkv) umma_commit(&sm.bar_o_full[t]);
+            if (t == kNQ - 1) umma_commit(&sm.bar_v_empty[pst]);
           }
           if (j < nkv) {
+            if (t == 0) {
+              ok = mbar_wait(&sm.bar_k_full[st], (j >> 1) & 1, &sm.abort);
+              if (!ok) break;
+              tc_fence_after_sync();
+            }
             // S_t = Q_t . K(j)^T, both K-major with 128-byte swizzle
 #pragma unroll
             for (int ks = 0; ks < kD / 16; ++ks) {
@@ -227,11 +224,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                       ks > 0 ? 1u : 0u);
             }
             umma_commit(&sm.bar_s_full[t]);
+            if (t == kNQ - 1) umma_commit(&sm.bar_k_empty[st]);
+            if (t == 0) {
+              // V(j) feeds the P.V products of the next KV step; it was issued long before
+              ok = mbar_wait(&sm.bar_v_full[st], (j >> 1) & 1, &sm.abort);
+              if (!ok) break;
+            }
           }
         }
-        if (!ok) break;
-        if (j < nkv) umma_commit(&sm.bar_k_empty[st]);
-        if (j > 0) umma_commit(&sm.bar_v_empty[(j - 1) & 1]);
       }
       if (!ok) raise_abort(sm, status, 20);
       // all tensor-core work of this CTA must finish before tensor memory is released
@@ -309,12 +309,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       // row maximum: four independent 3-input max chains
       float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
 #pragma unroll
-      for (int c = 4; c < kBN; c += 8) {
+      for (int c = 4; c + 8 <= kBN; c += 8) {
         mx0 = fmax3(mx0, s[c], s[c + 1]);
         mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
         mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
         mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
       }
+      mx0 = fmax3(mx0, s[kBN - 4], s[kBN - 3]);
+      mx1 = fmax3(mx1, s[kBN - 2], s[kBN - 1]);
       const float m_tile = fmax3(mx0, mx1, fmaxf(mx2, mx3)) * scale_log2;
       float alpha = 1.0f;
       bool rescaled = false;
