@@ -19,6 +19,10 @@ Everything here is written from the paper's definitions:
 * §6.1: entropy-ordered greedy unmasking (Shannon entropy of p).
 * §5.3: uncertainty u(j) = -log p_j(y_j), Score(j) = u (1 + d_in)/(1 + d_out),
   top-k seed selection over eligible positions.
+* §5.2 and §3 (one step's decisions): threshold drafting capped at B, the
+  Keep / Replace / ReMask revision of the previous seeds, the state update;
+  §5.3: the seed score on the updated state, the adaptive revision rate
+  |S_t| = ceil(sqrt(n_t pi_t)) and the exclusions from seed selection.
 
 Readings of points the paper leaves open (numbered as in the design notes):
 the cached inputs already hold the overridden memory K', V' (R1); the masked
@@ -29,7 +33,16 @@ of its corrected distribution (R6); out-of-range seeds are ignored and, among
 duplicates, the lowest slot wins (R7); ties in argmax / top-k go to the lower
 index (R9); entropy is natural-log Shannon entropy at temperature 1 (R10);
 without current tokens y = argmax (R11); absent d_in / d_out are 0 (R12);
-top-k takes the largest scores (R13).
+top-k takes the largest scores (R13). For the decision step: when no masked
+position passes the drafting threshold, the lowest-entropy one is drafted if
+the caller asks for guaranteed progress (R21); n_t, the mean and the empirical
+CDF run over every unmasked position of the updated state with a finite score,
+and the exclusions apply only to the selection (R22); |S_t| is further capped
+by the caller's seed capacity and the number of eligible positions (R23);
+"selected in the previous step" means S_{t-1} (R24); the seed score uses the
+uncertainty of the updated token, so a drafted or replaced position takes
+-log p(greedy token) (R25); drafting is limited to a caller-given set of
+positions, the active block of semi-autoregressive decoding (R26).
 
 Every function is pinned by ``tests/test_oracle_pins.py`` against closed forms,
 hand-worked fixtures, a library routine (torch float64 SDPA) and brute force.
@@ -293,3 +306,141 @@ def topk_margin(score: np.ndarray, n_seq: int, k: int, eligible=None):
         if len(vals) > k:
             gaps[g] = vals[k - 1] - vals[k]
     return gaps
+
+
+# ----------------------------------------------------------------------------
+# One decoding step's decisions after scoring: §5.2 (threshold drafting with a
+# budget, the Keep / Replace / ReMask revision rule), §3 (state update) and
+# §5.3 (stability-aware seed score on the updated state, adaptive revision
+# rate |S_t| = ceil(sqrt(n_t pi_t)), exclusion of the previous seeds and of
+# positions that used up their ReMask budget).
+# ----------------------------------------------------------------------------
+
+FLAG_SEED = 1   # bit of the per-position flag byte: "in the seed set"
+
+
+def decide_sequence(conf, yhat, ent, u_cur, u_top, d_in, d_out, tok, flags, remask_cnt, draft_ok, *,
+                    tau: float, budget: int, m_remask: int, mask_id: int, min_one: bool, pos0: int,
+                    max_seeds: int):
+    """Decisions of one step for one sequence (rows = its response positions).
+
+    Per row i the scoring pass of this step supplies c_i = max_v p_i(v)
+    (``conf``), the greedy token (``yhat``), the entropy H_i (``ent``),
+    u_cur = -log p_i(y_i^(t-1)) for the current token and u_top = -log p_i(yhat_i).
+    ``tok`` holds y^(t-1) with ``mask_id`` for [MASK]; bit FLAG_SEED of
+    ``flags`` marks S_{t-1}; ``remask_cnt`` counts each position's ReMasks so
+    far; ``draft_ok`` marks the positions the drafting rule may unmask (the
+    active block of semi-autoregressive decoding); d_in / d_out are the
+    influence terms of the seed score (None = 0).
+
+    The seed score is formed in the floating-point type of ``u_cur`` / ``u_top``
+    as (u * (1 + d_in)) / (1 + d_out); every comparison that follows (the
+    threshold, the orderings, the mean of the adaptive rate) is exact on those
+    values (the mean is a Fraction).
+
+    Returns a dict: tok, remask_cnt, flags (new arrays), drafted / kept /
+    replaced / remasked (sorted index lists), score (per row, -inf where the
+    new state is [MASK] or the score is not finite), n_t, n_above, n_select,
+    seeds (positions pos0 + i in selection order).
+    """
+    from fractions import Fraction
+
+    n = len(tok)
+    tok = np.asarray(tok, dtype=np.int64)
+    flags = np.asarray(flags, dtype=np.int64)
+    remask_cnt = np.asarray(remask_cnt, dtype=np.int64)
+    conf = np.asarray(conf)
+    dtype = np.asarray(u_cur).dtype.type
+
+    # masked / unmasked sets at the start of the step (§3)
+    masked = [i for i in range(n) if tok[i] == mask_id]
+    unmasked = [i for i in range(n) if tok[i] != mask_id]
+    seeds_prev = [i for i in unmasked if flags[i] & FLAG_SEED]
+
+    # drafting (§5.2): masked positions whose confidence exceeds tau, at most
+    # `budget` of them, the largest confidences kept (ties to the lower index)
+    draftable = [i for i in masked if draft_ok is None or draft_ok[i]]
+    over = [i for i in draftable if conf[i] > tau]
+    over.sort(key=lambda i: (-float(conf[i]), i))
+    drafted = sorted(over[:max(budget, 0)])
+    if not drafted and min_one and draftable:
+        # guaranteed progress: the lowest-entropy masked position (§6.1)
+        drafted = [min(draftable, key=lambda i: (float(ent[i]), i))]
+
+    # revision of the previous seeds (§5.2): Keep / Replace / ReMask
+    kept, replaced, remasked = [], [], []
+    for i in seeds_prev:
+        if yhat[i] == tok[i]:
+            kept.append(i)
+        elif conf[i] > tau:
+            replaced.append(i)
+        else:
+            remasked.append(i)
+
+    # state update (§3)
+    new_tok = tok.copy()
+    new_rc = remask_cnt.copy()
+    for i in drafted + replaced:
+        new_tok[i] = yhat[i]
+    for i in remasked:
+        new_tok[i] = mask_id
+        new_rc[i] += 1
+    changed = set(drafted) | set(replaced)
+
+    # seed score on the updated state (§5.3): u = -log p(y^(t))
+    score = np.full(n, -np.inf)
+    scored = []
+    one = dtype(1)
+    for i in range(n):
+        if new_tok[i] == mask_id:
+            continue
+        u = dtype(u_top[i]) if i in changed else dtype(u_cur[i])
+        din = dtype(0) if d_in is None else dtype(d_in[i])
+        dout = dtype(0) if d_out is None else dtype(d_out[i])
+        s = dtype(dtype(u * dtype(one + din)) / dtype(one + dout))
+        if np.isfinite(s):
+            score[i] = s
+            scored.append(i)
+
+    # adaptive revision rate (§5.3): n_t, the empirical CDF at the mean, pi_t
+    n_t = len(scored)
+    n_select = 0
+    n_above = 0
+    if n_t > 0:
+        vals = {i: Fraction(float(score[i])) for i in scored}
+        mean = sum(vals.values()) / n_t
+        F = Fraction(sum(1 for i in scored if vals[i] <= mean), n_t)
+        pi = 1 - F
+        n_above = int(n_t * pi)                  # n_t * pi_t is a whole number
+        n_select = math.isqrt(n_above)
+        if n_select * n_select < n_above:
+            n_select += 1                        # ceil(sqrt(n_t pi_t))
+    n_select = min(n_select, max_seeds)
+
+    # selection: previous seeds and positions at the ReMask budget are excluded
+    prev = set(seeds_prev)
+    eligible = [i for i in scored if i not in prev and new_rc[i] < m_remask]
+    eligible.sort(key=lambda i: (-float(score[i]), i))
+    chosen = eligible[:n_select]
+
+    new_flags = flags & ~FLAG_SEED
+    for i in chosen:
+        new_flags[i] |= FLAG_SEED
+    return dict(tok=new_tok, remask_cnt=new_rc, flags=new_flags, drafted=drafted, kept=sorted(kept),
+                replaced=sorted(replaced), remasked=sorted(remasked), score=score, n_t=n_t, n_above=n_above,
+                n_select=len(chosen), seeds=[pos0 + i for i in chosen])
+
+
+def decide_step(conf, yhat, ent, u_cur, u_top, d_in, d_out, tok, flags, remask_cnt, draft_ok, n_seq: int,
+                **params):
+    """decide_sequence over the n_seq equal consecutive segments of N rows."""
+    N = len(tok)
+    per = N // n_seq
+    outs = []
+    for g in range(n_seq):
+        sl = slice(g * per, (g + 1) * per)
+        pick = (lambda a: None if a is None else np.asarray(a)[sl])
+        outs.append(decide_sequence(pick(conf), pick(yhat), pick(ent), pick(u_cur), pick(u_top), pick(d_in),
+                                    pick(d_out), pick(tok), pick(flags), pick(remask_cnt), pick(draft_ok),
+                                    **params))
+    return outs
