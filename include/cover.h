@@ -168,6 +168,66 @@ int cover_score_fwd_noalloc(const void* logits, int N, int V, int n_seq,
                             int32_t* topk_idx, float* topk_score, void* stream);
 
 /*
+ * One decoding step's decisions, fused behind the scoring pass
+ * (Section 5.2 "Threshold drafting" and the Keep / Replace / ReMask revision
+ * rule, Section 3 state update, Section 5.3 stability-aware seed score,
+ * adaptive revision rate and seed exclusions).
+ *
+ * The N rows split into n_seq equal segments (sequences); row i of a segment
+ * is response position pos0 + i. Per row the scoring pass computes c = max p,
+ * y_hat = argmax p (ties to the lower index) and H exactly as
+ * cover_score_fwd, and u = -log p(tok) for the current token. Then, per
+ * segment (state arrays updated in place):
+ *   1. Drafting: among rows with tok == mask_id and draft_ok != 0 (all such
+ *      rows when draft_ok is NULL), those with c > tau_draft; if more than
+ *      draft_budget, the largest c are kept (ties to the lower index). If none
+ *      is drafted and min_one != 0, the allowed masked row with the lowest H is
+ *      drafted (ties to the lower index). Drafted rows take tok = y_hat.
+ *   2. Revision of the previous seeds (rows with flag bit COVER_FLAG_SEED set
+ *      and tok != mask_id): Keep if y_hat == tok; else Replace (tok = y_hat)
+ *      if c > tau_draft; else ReMask (tok = mask_id, remask_cnt + 1, saturating
+ *      at 255).
+ *   3. Seed score of every unmasked row of the updated state, in fp32:
+ *      score = (u * (1 + d_in)) / (1 + d_out), with u = ln Z = -log c for
+ *      drafted and replaced rows and the current token's u otherwise (NULL
+ *      d_in / d_out = 0). Masked rows and non-finite scores get -INFINITY.
+ *   4. Adaptive revision rate: n_t = rows with a finite score, n_above = rows
+ *      with n_t * score > sum of the scores (fp64; this is n_t * pi_t),
+ *      k = min(ceil(sqrt(n_above)), max_seeds).
+ *   5. New seeds: the k highest-scoring rows (ties to the lower index) among
+ *      the scored rows that were not previous seeds and have
+ *      remask_cnt < remask_budget; fewer if fewer are eligible. Their flag bit
+ *      COVER_FLAG_SEED is set and every other row's is cleared (other flag bits
+ *      are kept); seed_idx[seg, 0..n_seeds) lists their positions pos0 + i in
+ *      order, the rest of the row is -1, so it can be passed to
+ *      cover_attn_fwd as the next step's seed_idx with n_seeds = max_seeds.
+ *
+ * logits   bf16 [N, V] row-major, 16-byte aligned (device).
+ * d_in, d_out, draft_ok: [N] or NULL (device).
+ * tok      int32 [N] (device, in/out); flags, remask_cnt uint8 [N] (in/out).
+ * maxprob, entropy, score float [N]; argmax int32 [N] (device, out).
+ * seed_idx int32 [n_seq, max_seeds] (device, out; may be NULL if max_seeds is
+ *          0); n_seeds int32 [n_seq] (out); stats int32 [n_seq, 6] or NULL:
+ *          drafted, kept, replaced, remasked, n_t, n_above per segment.
+ * workspace: cover_decide_workspace_bytes(N, n_seq) bytes of device memory,
+ *          16-byte aligned, zero-filled before its first use; it is left ready
+ *          for the next call on the same stream.
+ * Errors: COVER_ERR_INVALID_ARG for a NULL required pointer, N, V or n_seq < 1,
+ * N % n_seq != 0, N / n_seq > 4096, draft_budget, remask_budget or max_seeds
+ * < 0, or a misaligned pointer. COVER_ERR_CUDA for a launch failure.
+ */
+#define COVER_FLAG_SEED 1
+size_t cover_decide_workspace_bytes(int N, int n_seq);
+int cover_score_decide_fwd(const void* logits, int N, int V, int n_seq,
+                           const float* d_in, const float* d_out, const uint8_t* draft_ok,
+                           float tau_draft, int draft_budget, int remask_budget, int mask_id,
+                           int min_one, int pos0, int max_seeds,
+                           int32_t* tok, uint8_t* flags, uint8_t* remask_cnt,
+                           float* maxprob, float* entropy, int32_t* argmax, float* score,
+                           int32_t* seed_idx, int32_t* n_seeds, int32_t* stats,
+                           void* workspace, void* stream);
+
+/*
  * Synchronises `stream`, then returns and clears the current device's status
  * word: COVER_OK, or COVER_ERR_DEVICE_TIMEOUT if a kernel gave up on a
  * bounded wait since the last call. Returns COVER_ERR_CUDA if the

@@ -186,6 +186,59 @@ def cover_score_fwd_noalloc(logits, n_seq: int, topk: int, *, cur_tok=None, d_in
     return out
 
 
+def cover_decide_workspace_bytes(N: int, n_seq: int) -> int:
+    return int(_lib.load().cover_decide_workspace_bytes(int(N), int(n_seq)))
+
+
+def decide_workspace(N: int, n_seq: int, device=None) -> torch.Tensor:
+    """A zero-filled workspace for cover_score_decide_fwd (reusable across calls on one stream)."""
+    nbytes = cover_decide_workspace_bytes(N, n_seq)
+    return torch.zeros((max(nbytes, 16) + 15) // 16, 4, dtype=torch.int32, device=device or "cuda")
+
+
+def cover_score_decide_fwd(logits, n_seq: int, tok, flags, remask_cnt, *, tau_draft: float, draft_budget: int,
+                           remask_budget: int, mask_id: int, min_one: bool = True, pos0: int = 0,
+                           max_seeds: int = 0, d_in=None, d_out=None, draft_ok=None, workspace=None, out=None,
+                           stream=None):
+    """Scoring fused with one decoding step's decisions (drafting, revision, seed selection).
+
+    tok (int32 [N]), flags and remask_cnt (uint8 [N]) are updated in place.
+    Returns a dict of CUDA tensors: maxprob, entropy, argmax, score [N];
+    seed_idx [n_seq, max_seeds] (positions, -1 padded), n_seeds [n_seq] and
+    stats [n_seq, 6] (drafted, kept, replaced, remasked, n_t, n_above).
+    """
+    _need(logits, "logits", torch.bfloat16, 2)
+    N, V = logits.shape
+    dev = logits.device
+    _need(tok, "tok", torch.int32, 1)
+    _need(flags, "flags", torch.uint8, 1)
+    _need(remask_cnt, "remask_cnt", torch.uint8, 1)
+    for name, t, dt in (("d_in", d_in, torch.float32), ("d_out", d_out, torch.float32),
+                        ("draft_ok", draft_ok, torch.uint8)):
+        if t is not None:
+            _need(t, name, dt, 1)
+    if out is None:
+        out = dict(
+            maxprob=torch.empty(N, dtype=torch.float32, device=dev),
+            entropy=torch.empty(N, dtype=torch.float32, device=dev),
+            argmax=torch.empty(N, dtype=torch.int32, device=dev),
+            score=torch.empty(N, dtype=torch.float32, device=dev),
+            seed_idx=torch.empty((n_seq, max(max_seeds, 0)), dtype=torch.int32, device=dev),
+            n_seeds=torch.empty(n_seq, dtype=torch.int32, device=dev),
+            stats=torch.empty((n_seq, 6), dtype=torch.int32, device=dev),
+        )
+    if workspace is None:
+        workspace = decide_workspace(N, n_seq, dev)
+    code = _lib.load().cover_score_decide_fwd(
+        _ptr(logits), N, V, n_seq, _ptr(d_in), _ptr(d_out), _ptr(draft_ok), float(tau_draft), int(draft_budget),
+        int(remask_budget), int(mask_id), 1 if min_one else 0, int(pos0), int(max_seeds),
+        _ptr(tok), _ptr(flags), _ptr(remask_cnt), _ptr(out["maxprob"]), _ptr(out["entropy"]), _ptr(out["argmax"]),
+        _ptr(out["score"]), _ptr(out["seed_idx"]) if max_seeds > 0 else None, _ptr(out["n_seeds"]),
+        _ptr(out["stats"]), _ptr(workspace), _stream(stream))
+    _lib.check("cover_score_decide_fwd", code)
+    return out
+
+
 def cover_device_status(stream=None) -> int:
     """Synchronise the stream; return and clear the device status word (0 = OK)."""
     return int(_lib.load().cover_device_status(_stream(stream)))

@@ -134,6 +134,43 @@ int cover_score_fwd_noalloc(const void* logits, int N, int V, int n_seq, const i
   return cover::launch_score_noalloc(a, st, static_cast<cudaStream_t>(stream));
 }
 
+size_t cover_decide_workspace_bytes(int N, int n_seq) {
+  if (N < 1 || n_seq < 1) return 0;
+  // per-segment counters, then u and ln Z per row
+  const size_t counters = (sizeof(uint32_t) * static_cast<size_t>(n_seq) + 15) & ~static_cast<size_t>(15);
+  return counters + 2 * sizeof(float) * static_cast<size_t>(N);
+}
+
+int cover_score_decide_fwd(const void* logits, int N, int V, int n_seq, const float* d_in, const float* d_out,
+                           const uint8_t* draft_ok, float tau_draft, int draft_budget, int remask_budget,
+                           int mask_id, int min_one, int pos0, int max_seeds, int32_t* tok, uint8_t* flags,
+                           uint8_t* remask_cnt, float* maxprob, float* entropy, int32_t* argmax, float* score,
+                           int32_t* seed_idx, int32_t* n_seeds, int32_t* stats, void* workspace, void* stream) {
+  if (logits == nullptr || tok == nullptr || flags == nullptr || remask_cnt == nullptr || maxprob == nullptr ||
+      entropy == nullptr || argmax == nullptr || score == nullptr || n_seeds == nullptr || workspace == nullptr)
+    return COVER_ERR_INVALID_ARG;
+  if (N < 1 || V < 1 || n_seq < 1 || N % n_seq != 0 || N / n_seq > 4096) return COVER_ERR_INVALID_ARG;
+  if (draft_budget < 0 || remask_budget < 0 || max_seeds < 0) return COVER_ERR_INVALID_ARG;
+  if (max_seeds > 0 && seed_idx == nullptr) return COVER_ERR_INVALID_ARG;
+  if (!aligned(logits, 16) || !aligned(workspace, 16) || !aligned(tok, 4) || !aligned(maxprob, 4) ||
+      !aligned(entropy, 4) || !aligned(argmax, 4) || !aligned(score, 4) || !aligned(n_seeds, 4))
+    return COVER_ERR_INVALID_ARG;
+  if ((seed_idx != nullptr && !aligned(seed_idx, 4)) || (stats != nullptr && !aligned(stats, 4)) ||
+      (d_in != nullptr && !aligned(d_in, 4)) || (d_out != nullptr && !aligned(d_out, 4)))
+    return COVER_ERR_INVALID_ARG;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  const size_t counters_bytes = (sizeof(uint32_t) * static_cast<size_t>(n_seq) + 15) & ~static_cast<size_t>(15);
+  float* ws_u = reinterpret_cast<float*>(ws + counters_bytes);
+  float* ws_lnz = ws_u + N;
+  cover::ScoreArgs a{logits, N, V, n_seq, nullptr, d_in, d_out, nullptr, 0, maxprob, entropy, argmax, score,
+                     nullptr, nullptr, reinterpret_cast<uint32_t*>(ws)};
+  cover::DecideArgs d{draft_ok, tau_draft, draft_budget, remask_budget, mask_id, min_one != 0 ? 1 : 0, pos0,
+                      max_seeds, tok, flags, remask_cnt, seed_idx, n_seeds, stats, ws_u, ws_lnz};
+  return cover::launch_score_decide(a, d, st, static_cast<cudaStream_t>(stream));
+}
+
 int cover_device_status(void* stream) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int* st = status_block();

@@ -46,6 +46,30 @@ struct ScoreArgs {
 
 int launch_score(const ScoreArgs& a, int* status, cudaStream_t stream);
 
+// One decoding step's decisions, run by the last CTA of each segment after the
+// per-row scoring (a.topk, a.eligible, a.cur_tok, a.topk_idx and a.topk_score
+// are unused; a.score receives the seed scores of the updated state).
+struct DecideArgs {
+  const uint8_t* draft_ok;   // [N] or null (every masked row may be drafted)
+  float tau;                 // drafting / Replace threshold on the confidence
+  int budget;                // at most this many drafted rows per segment
+  int remask_budget;         // rows with this many ReMasks are not selected
+  int mask_id;               // token id of [MASK]
+  int min_one;               // draft the lowest-entropy masked row when none passes tau
+  int pos0;                  // position of a segment's first row
+  int max_seeds;             // seed capacity per segment
+  int32_t* tok;              // [N] in: current tokens, out: updated tokens
+  uint8_t* flags;            // [N] bit 0 in: previous seeds, out: new seeds
+  uint8_t* remask_cnt;       // [N] in / out
+  int32_t* seed_idx;         // [n_seq, max_seeds] positions, -1 padded
+  int32_t* n_seeds;          // [n_seq]
+  int32_t* stats;            // [n_seq, 6] or null
+  float* ws_u;               // [N] workspace: u of the current token
+  float* ws_lnz;             // [N] workspace: ln Z (= u of the greedy token)
+};
+constexpr int kDecideStats = 6;   // drafted, kept, replaced, remasked, n_t, n_above
+int launch_score_decide(const ScoreArgs& a, const DecideArgs& d, int* status, cudaStream_t stream);
+
 // Same as launch_score, with the counters in a fixed device array of the
 // library (a.counters is ignored). Returns -1 if a.n_seq > kNoAllocMaxSegments.
 constexpr int kNoAllocMaxSegments = 4096;

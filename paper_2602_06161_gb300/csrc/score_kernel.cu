@@ -17,6 +17,14 @@
 // eligible rows by (score descending, index ascending) with a bitonic sort of
 // 64-bit keys in shared memory and writes the first k.
 //
+// Decision step (cover_score_decide_fwd, Sections 5.2, 3 and 5.3): the row
+// pass keeps u of the current token and ln Z (= u of the greedy token) in a
+// workspace; the last CTA of a segment then drafts the most confident masked
+// rows above the threshold (at most B), applies Keep / Replace / ReMask to the
+// previous seeds, scores the updated state, counts the scores above their mean
+// (n_t pi_t), and selects ceil(sqrt(n_t pi_t)) new seeds among the rows that
+// were not seeds and have ReMasks left, with the same 64-bit key sort.
+//
 // Two ways to stream a row:
 //  * score_bulk_kernel (rows 16-byte aligned, V % 8 == 0): a producer warp
 //    issues cp.async.bulk copies of 16 KB chunks into a 3-stage shared-memory
@@ -201,7 +209,7 @@ __device__ __forceinline__ RowOut row_reduce(const RowAcc& a, float* red_m, int*
 __device__ __forceinline__ bool row_write(const RowOut& r, int n, const uint16_t* row, int V, int per_seq,
                                           const int32_t* cur_tok, const float* d_in, const float* d_out, int topk,
                                           float* maxprob, float* entropy, int32_t* argmax, float* score,
-                                          uint32_t* counters) {
+                                          uint32_t* counters, float* ws_u = nullptr, float* ws_lnz = nullptr) {
   const float Zf = static_cast<float>(r.Z);
   const float lnZ = logf(Zf);
   const float H = lnZ - 0.6931471805599453f * static_cast<float>(r.S / r.Z);
@@ -216,12 +224,220 @@ __device__ __forceinline__ bool row_write(const RowOut& r, int n, const uint16_t
   maxprob[n] = 1.0f / Zf;
   entropy[n] = H;
   argmax[n] = r.yhat;
-  score[n] = u * (1.0f + din) / (1.0f + dout);
-  if (topk <= 0) return false;
+  if (ws_u != nullptr) {
+    // decision step: the seed score is formed after the state update
+    ws_u[n] = u;
+    ws_lnz[n] = lnZ;
+  } else {
+    score[n] = u * (1.0f + din) / (1.0f + dout);
+    if (topk <= 0) return false;
+  }
   __threadfence();
   const unsigned seg = static_cast<unsigned>(n / per_seq);
   const unsigned old = atomicInc(counters + seg, static_cast<unsigned>(per_seq - 1));
   return old == static_cast<unsigned>(per_seq - 1);
+}
+
+struct ScoreParams {
+  const uint16_t* logits;
+  int V, per_seq;
+  const int32_t* cur_tok;
+  const float* d_in;
+  const float* d_out;
+  const uint8_t* eligible;
+  int topk, sort_n;
+  float* maxprob;
+  float* entropy;
+  int32_t* argmax;
+  float* score;
+  int32_t* topk_idx;
+  float* topk_score;
+  uint32_t* counters;
+  int decide;          // 1: run the decision step instead of the top-k
+  DecideArgs dec;
+};
+
+// Descending bitonic sort of n (a power of two) 64-bit keys in shared memory;
+// all threads of the CTA call it.
+__device__ __forceinline__ void bitonic_sort_desc(uint64_t* keys, int n) {
+  const int tid = threadIdx.x, nt = blockDim.x;
+  for (int k = 2; k <= n; k <<= 1) {
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      for (int i = tid; i < n; i += nt) {
+        const int p = i ^ j;
+        if (p > i) {
+          const uint64_t x = keys[i], y = keys[p];
+          const bool desc = (i & k) == 0;
+          if (desc ? (x < y) : (x > y)) {
+            keys[i] = y;
+            keys[p] = x;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+}
+
+// Sum over the CTA (blockDim a multiple of 32); every thread gets the total,
+// added in the same order everywhere. scratch: 32 entries.
+template <typename T>
+__device__ __forceinline__ T block_sum(T v, T* scratch) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();
+  if (lane == 0) scratch[warp] = v;
+  __syncthreads();
+  T t = 0;
+  for (int w = 0; w < nw; ++w) t += scratch[w];
+  return t;
+}
+
+// key of row i ordered by value descending, then index ascending; 0 = no row
+__device__ __forceinline__ uint64_t rank_key(float v, int i) {
+  return (static_cast<uint64_t>(order_key(v)) << 32) | (0xffffffffu - static_cast<uint32_t>(i));
+}
+__device__ __forceinline__ int rank_key_row(uint64_t key) {
+  return static_cast<int>(0xffffffffu - static_cast<uint32_t>(key));
+}
+
+// The last CTA of a segment: one decoding step's decisions for that sequence.
+// Rows written by other CTAs are read through L2 (__ldcg).
+__device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n, const ScoreParams& P) {
+  __shared__ unsigned long long s_fallback;
+  __shared__ int s_ri[32];
+  __shared__ double s_rd[32];
+  __threadfence();
+  const DecideArgs& d = P.dec;
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int base = seg * per_seq;
+  if (tid == 0) s_fallback = ~0ull;
+  __syncthreads();
+
+  // Section 5.2 drafting: masked rows in the allowed set whose confidence exceeds tau
+  int ncand = 0;
+  for (int i = tid; i < sort_n; i += nt) {
+    uint64_t key = 0;
+    if (i < per_seq) {
+      const int n = base + i;
+      if (d.tok[n] == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0)) {
+        const float c = __ldcg(P.maxprob + n);
+        if (c > d.tau) {
+          key = rank_key(c, i);
+          ++ncand;
+        }
+        if (d.min_one) {
+          // lowest entropy, then lowest index
+          const uint64_t fb = (static_cast<uint64_t>(order_key(__ldcg(P.entropy + n))) << 32) | static_cast<uint32_t>(i);
+          atomicMin(&s_fallback, static_cast<unsigned long long>(fb));
+        }
+      }
+    }
+    keys[i] = key;
+  }
+  ncand = block_sum(ncand, s_ri);
+  bitonic_sort_desc(keys, sort_n);
+  int n_drafted = min(ncand, d.budget);
+  const bool fallback = n_drafted == 0 && d.min_one && s_fallback != ~0ull;
+  for (int t = tid; t < (fallback ? 1 : n_drafted); t += nt) {
+    const int n = base + (fallback ? static_cast<int>(static_cast<uint32_t>(s_fallback)) : rank_key_row(keys[t]));
+    // a drafted row takes its greedy token, whose uncertainty is ln Z
+    d.tok[n] = __ldcg(P.argmax + n);
+    d.ws_u[n] = __ldcg(d.ws_lnz + n);
+    d.flags[n] = static_cast<uint8_t>(d.flags[n] & ~1u);
+  }
+  if (fallback) n_drafted = 1;
+  __syncthreads();
+
+  // Section 5.2 revision of the previous seeds, Section 3 state update, Section 5.3 seed score
+  int kept = 0, replaced = 0, remasked = 0, n_t = 0;
+  double total = 0.0;
+  for (int i = tid; i < sort_n; i += nt) {
+    uint64_t key = 0;
+    if (i < per_seq) {
+      const int n = base + i;
+      int y = d.tok[n];
+      const uint8_t fl = d.flags[n];
+      int rc = d.remask_cnt[n];
+      const bool was_seed = (fl & 1u) != 0 && y != d.mask_id;
+      float u = __ldcg(d.ws_u + n);
+      if (was_seed) {
+        const int yh = __ldcg(P.argmax + n);
+        if (yh == y) {
+          ++kept;
+        } else if (__ldcg(P.maxprob + n) > d.tau) {
+          ++replaced;
+          y = yh;
+          u = __ldcg(d.ws_lnz + n);
+        } else {
+          ++remasked;
+          y = d.mask_id;
+          rc = min(rc + 1, 255);
+        }
+        d.tok[n] = y;
+        d.remask_cnt[n] = static_cast<uint8_t>(rc);
+      }
+      d.flags[n] = static_cast<uint8_t>(fl & ~1u);
+      float s = -INFINITY;
+      if (y != d.mask_id) {
+        const float din = P.d_in != nullptr ? P.d_in[n] : 0.0f;
+        const float dout = P.d_out != nullptr ? P.d_out[n] : 0.0f;
+        const float sc = u * (1.0f + din) / (1.0f + dout);
+        if (isfinite(sc)) {
+          s = sc;
+          ++n_t;
+          total += static_cast<double>(sc);
+          if (!was_seed && rc < d.remask_budget) key = rank_key(sc, i);
+        }
+      }
+      P.score[n] = s;
+    }
+    keys[i] = key;
+  }
+  kept = block_sum(kept, s_ri);
+  replaced = block_sum(replaced, s_ri);
+  remasked = block_sum(remasked, s_ri);
+  n_t = block_sum(n_t, s_ri);
+  total = block_sum(total, s_rd);
+
+  // Section 5.3 adaptive revision rate: n_t pi_t = #{ s_j > mean } = #{ n_t s_j > sum s }
+  int above = 0;
+  for (int i = tid; i < per_seq; i += nt) {
+    const float s = __ldcg(P.score + base + i);
+    if (s != -INFINITY && static_cast<double>(n_t) * static_cast<double>(s) > total) ++above;
+  }
+  above = block_sum(above, s_ri);
+  int k = 0;
+  while (k * k < above) ++k;   // ceil(sqrt(n_t pi_t))
+  k = min(k, d.max_seeds);
+
+  // selection: the k best eligible rows (keys written above)
+  bitonic_sort_desc(keys, sort_n);
+  int chosen = 0;
+  for (int t = tid; t < d.max_seeds; t += nt) {
+    int pos = -1;
+    if (t < k && t < sort_n && keys[t] != 0) {
+      const int i = rank_key_row(keys[t]);
+      pos = d.pos0 + i;
+      d.flags[base + i] = static_cast<uint8_t>(d.flags[base + i] | 1u);
+      ++chosen;
+    }
+    d.seed_idx[static_cast<size_t>(seg) * d.max_seeds + t] = pos;
+  }
+  chosen = block_sum(chosen, s_ri);
+  if (tid == 0) {
+    d.n_seeds[seg] = chosen;
+    if (d.stats != nullptr) {
+      int32_t* st = d.stats + static_cast<size_t>(seg) * kDecideStats;
+      st[0] = n_drafted;
+      st[1] = kept;
+      st[2] = replaced;
+      st[3] = remasked;
+      st[4] = n_t;
+      st[5] = above;
+    }
+  }
 }
 
 // The last CTA of a segment: top-k by (score desc, index asc) over eligible rows.
@@ -240,22 +456,7 @@ __device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_se
     keys[i] = key;
   }
   __syncthreads();
-  for (int k = 2; k <= sort_n; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = tid; i < sort_n; i += nt) {
-        const int p = i ^ j;
-        if (p > i) {
-          const uint64_t x = keys[i], y = keys[p];
-          const bool desc = (i & k) == 0;
-          if (desc ? (x < y) : (x > y)) {
-            keys[i] = y;
-            keys[p] = x;
-          }
-        }
-      }
-      __syncthreads();
-    }
-  }
+  bitonic_sort_desc(keys, sort_n);
   for (int t = tid; t < topk; t += nt) {
     const uint64_t key = keys[t];
     const bool valid = key != 0;
@@ -311,22 +512,6 @@ __device__ __forceinline__ void acc_batch(RowAcc& a, const uint4 (&w)[U], int i0
   kahan_add(a.s, a.sc, s0 + s1);
 }
 
-struct ScoreParams {
-  const uint16_t* logits;
-  int V, per_seq;
-  const int32_t* cur_tok;
-  const float* d_in;
-  const float* d_out;
-  const uint8_t* eligible;
-  int topk, sort_n;
-  float* maxprob;
-  float* entropy;
-  int32_t* argmax;
-  float* score;
-  int32_t* topk_idx;
-  float* topk_score;
-  uint32_t* counters;
-};
 
 // ---------------------------------------------------------------------------
 // register-load kernel (any V)
@@ -366,11 +551,16 @@ __global__ void __launch_bounds__(kThreads, 2) score_kernel(const ScoreParams P)
 
   const RowOut r = row_reduce<kWarps>(a, red_m, red_i, red_z, red_s);
   if (tid == 0)
-    s_last = row_write(r, n, row, V, P.per_seq, P.cur_tok, P.d_in, P.d_out, P.topk, P.maxprob, P.entropy, P.argmax,
-                       P.score, P.counters);
+    s_last = row_write(r, n, row, V, P.per_seq, P.decide ? P.dec.tok : P.cur_tok, P.d_in, P.d_out, P.topk,
+                       P.maxprob, P.entropy, P.argmax, P.score, P.counters, P.decide ? P.dec.ws_u : nullptr,
+                       P.decide ? P.dec.ws_lnz : nullptr);
   __syncthreads();
-  if (s_last)
-    segment_topk(keys, n / P.per_seq, P.per_seq, P.sort_n, P.topk, P.score, P.eligible, P.topk_idx, P.topk_score);
+  if (s_last) {
+    if (P.decide)
+      segment_decide(keys, n / P.per_seq, P.per_seq, P.sort_n, P);
+    else
+      segment_topk(keys, n / P.per_seq, P.per_seq, P.sort_n, P.topk, P.score, P.eligible, P.topk_idx, P.topk_score);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -466,23 +656,31 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
 
   const RowOut r = row_reduce<kConsumerWarps + 1>(a, red_m, red_i, red_z, red_s);
   if (tid == 0)
-    s_last = row_write(r, n, row, V, P.per_seq, P.cur_tok, P.d_in, P.d_out, P.topk, P.maxprob, P.entropy, P.argmax,
-                       P.score, P.counters);
+    s_last = row_write(r, n, row, V, P.per_seq, P.decide ? P.dec.tok : P.cur_tok, P.d_in, P.d_out, P.topk,
+                       P.maxprob, P.entropy, P.argmax, P.score, P.counters, P.decide ? P.dec.ws_u : nullptr,
+                       P.decide ? P.dec.ws_lnz : nullptr);
   __syncthreads();
-  if (s_last)
-    segment_topk(reinterpret_cast<uint64_t*>(ring), n / P.per_seq, P.per_seq, P.sort_n, P.topk, P.score,
-                 P.eligible, P.topk_idx, P.topk_score);
+  if (s_last) {
+    if (P.decide)
+      segment_decide(reinterpret_cast<uint64_t*>(ring), n / P.per_seq, P.per_seq, P.sort_n, P);
+    else
+      segment_topk(reinterpret_cast<uint64_t*>(ring), n / P.per_seq, P.per_seq, P.sort_n, P.topk, P.score,
+                   P.eligible, P.topk_idx, P.topk_score);
+  }
 }
 
 }  // namespace
 
-int launch_score(const ScoreArgs& a, int* status, cudaStream_t stream) {
+namespace {
+
+int launch_score_impl(const ScoreArgs& a, const DecideArgs* d, int* status, cudaStream_t stream) {
   const int per = a.N / a.n_seq;
   int sort_n = 1;
   while (sort_n < per) sort_n <<= 1;
   ScoreParams P{static_cast<const uint16_t*>(a.logits), a.V, per, a.cur_tok, a.d_in, a.d_out, a.eligible,
-                a.topk, sort_n, a.maxprob, a.entropy, a.argmax, a.score, a.topk_idx, a.topk_score, a.counters};
-  const size_t keys_bytes = a.topk > 0 ? sizeof(uint64_t) * static_cast<size_t>(sort_n) : 0;
+                a.topk, sort_n, a.maxprob, a.entropy, a.argmax, a.score, a.topk_idx, a.topk_score, a.counters,
+                d != nullptr ? 1 : 0, d != nullptr ? *d : DecideArgs{}};
+  const size_t keys_bytes = (a.topk > 0 || d != nullptr) ? sizeof(uint64_t) * static_cast<size_t>(sort_n) : 0;
   const bool aligned_rows = (a.V % 8) == 0 && (reinterpret_cast<uintptr_t>(a.logits) % 16) == 0;
   if (aligned_rows) {
     const size_t smem = std::max(keys_bytes, static_cast<size_t>(kRingStages) * kChunkBytes);
@@ -498,6 +696,16 @@ int launch_score(const ScoreArgs& a, int* status, cudaStream_t stream) {
     score_kernel<<<a.N, kThreads, keys_bytes, stream>>>(P);
   }
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
+}
+
+}  // namespace
+
+int launch_score(const ScoreArgs& a, int* status, cudaStream_t stream) {
+  return launch_score_impl(a, nullptr, status, stream);
+}
+
+int launch_score_decide(const ScoreArgs& a, const DecideArgs& d, int* status, cudaStream_t stream) {
+  return launch_score_impl(a, &d, status, stream);
 }
 
 // ---------------------------------------------------------------------------

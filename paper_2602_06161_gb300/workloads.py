@@ -19,6 +19,17 @@ datasets are used, synthetic tensors of the same shapes stand in):
 * Logits come from a separate ``default_rng(seed + 1)``: N(0, 2) means
   variance 2 (standard deviation sqrt(2)). Spiked rows get +8 added to one
   uniformly chosen vocabulary entry before bf16 rounding.
+* Decision-step state (make_decide_inputs, ``default_rng(seed + 2)``): per
+  sequence of ``per`` response positions an active block of ``block_len``
+  positions (64 for LLaDA-shaped, 32 for Dream-shaped workloads, §6.1) starts
+  at a uniformly drawn multiple of ``block_len``; positions before it hold
+  tokens, positions inside it are masked with probability 1/2, positions after
+  it are masked. ceil(sqrt(unmasked)) unmasked positions carry the
+  previous-seed flag; unmasked positions have ReMask counts uniform in
+  [0, m_remask]. [MASK] is token V - 128. Logits are N(0, var) plus, on one
+  token per row, a spike uniform in [0, max_spike): the current token with
+  probability 1/2 for previous seeds, else a uniform token. d_in and d_out are
+  uniform in [0, 2).
 * Seed positions: "uniform" draws S distinct positions from [lo, hi) without
   replacement, in draw order (slot s <-> draw s). "runs" draws the starts of
   ``n_runs`` contiguous runs uniformly from [lo, hi - run_len] and rejects a
@@ -200,6 +211,67 @@ def make_score_inputs(N: int, V: int, n_seq: int, topk: int, *, seed: int = 0, v
     return inp
 
 
+@dataclasses.dataclass
+class DecideInputs:
+    """Logits and decoding state for one step of the decision epilogue."""
+    N: int
+    V: int
+    n_seq: int
+    mask_id: int
+    logits: np.ndarray       # uint16 bf16 bits [N, V]
+    tok: np.ndarray          # int32 [N]; mask_id marks [MASK]
+    flags: np.ndarray        # uint8 [N]; bit 0 marks the previous seeds
+    remask_cnt: np.ndarray   # uint8 [N]
+    draft_ok: np.ndarray     # uint8 [N]; the active block
+    d_in: np.ndarray         # float32 [N]
+    d_out: np.ndarray        # float32 [N]
+
+    def logits_f64(self, rows=None) -> np.ndarray:
+        b = self.logits if rows is None else self.logits[rows]
+        return bf16_bits_to_f64(b)
+
+
+def make_decide_inputs(N: int, V: int, n_seq: int, *, seed: int = 0, block_len: int = 64, var: float = 2.0,
+                       max_spike: float = 16.0, m_remask: int = 5) -> DecideInputs:
+    """Draw one decoding step's state and its logits (recipe in the module docstring)."""
+    rng = np.random.default_rng(seed + 2)
+    per = N // n_seq
+    mask_id = V - 128 if V > 128 else V - 1
+    tok = rng.integers(0, V - 1, size=N).astype(np.int32)
+    tok[tok >= mask_id] += 1                              # real tokens never equal [MASK]
+    flags = np.zeros(N, dtype=np.uint8)
+    remask = np.zeros(N, dtype=np.uint8)
+    draft_ok = np.zeros(N, dtype=np.uint8)
+    n_blocks = max(1, -(-per // block_len))
+    for g in range(n_seq):
+        base = g * per
+        lo = int(rng.integers(0, n_blocks)) * block_len
+        hi = min(per, lo + block_len)
+        in_block = rng.uniform(size=hi - lo) < 0.5
+        seg = tok[base:base + per]
+        seg[hi:] = mask_id
+        seg[lo:hi][in_block] = mask_id
+        draft_ok[base + lo:base + hi] = 1
+        unmasked = np.nonzero(seg != mask_id)[0]
+        if len(unmasked):
+            k = int(math.ceil(math.sqrt(len(unmasked))))
+            pick = rng.choice(unmasked, size=k, replace=False)
+            flags[base + pick] = 1
+            remask[base + unmasked] = rng.integers(0, m_remask + 1, size=len(unmasked))
+    x = rng.standard_normal((N, V), dtype=np.float32)
+    x *= np.float32(math.sqrt(var))
+    spike_tok = rng.integers(0, V, size=N)
+    keep = (flags == 1) & (rng.uniform(size=N) < 0.5)
+    spike_tok[keep] = tok[keep]
+    spike = rng.uniform(0.0, max_spike, size=N).astype(np.float32)
+    x[np.arange(N), spike_tok] += spike
+    logits = f32_to_bf16_bits(x)
+    del x
+    d_in = rng.uniform(0.0, 2.0, size=N).astype(np.float32)
+    d_out = rng.uniform(0.0, 2.0, size=N).astype(np.float32)
+    return DecideInputs(N, V, n_seq, mask_id, logits, tok, flags, remask, draft_ok, d_in, d_out)
+
+
 # ----------------------------------------------------------------------------
 # The five named workloads
 # ----------------------------------------------------------------------------
@@ -224,6 +296,7 @@ class Workload:
     score_n_seq: Optional[int] = None
     score_topk: Optional[int] = None
     score_spike_frac: float = 0.0
+    decide_block: int = 64
     seed: int = 0
 
     @property
@@ -243,6 +316,13 @@ class Workload:
                                  seed=self.seed, spike_frac=self.score_spike_frac)
 
 
+    def decide_inputs(self) -> Optional[DecideInputs]:
+        if self.score_N is None:
+            return None
+        return make_decide_inputs(self.score_N, self.score_V, self.score_n_seq, seed=self.seed,
+                                  block_len=self.decide_block)
+
+
 WORKLOADS = {
     # tiny fp32 check
     "tiny_f32_l64": Workload("tiny_f32_l64", 1, 2, 2, 64, 64, 4, "f32", 32, 64),
@@ -252,7 +332,7 @@ WORKLOADS = {
     # Dream-7B-shaped GQA layer 28/4 x 128, L = 512 + 512, plus vocab-152064 scoring
     "dream_gqa_l1024": Workload("dream_gqa_l1024", 1, 28, 4, 1024, 128, 32, "bf16", 512, 1024,
                                 score_N=1024, score_V=152064, score_n_seq=1, score_topk=32,
-                                score_spike_frac=0.05),
+                                score_spike_frac=0.05, decide_block=32),
     # batched LLaDA-shaped, B=8, L=2048, plus vocab-126464 scoring of 8 x 256 rows
     "llada_b8_l2048": Workload("llada_b8_l2048", 8, 32, 32, 2048, 128, 64, "bf16", 1024, 2048,
                                score_N=8 * 256, score_V=126464, score_n_seq=8, score_topk=64),

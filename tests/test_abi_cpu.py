@@ -100,3 +100,27 @@ def test_debug_invalid_args(lib):
 def test_workspace_bytes(lib):
     assert lib.cover_score_workspace_bytes(8) == 32
     assert lib.cover_score_workspace_bytes(0) == 0
+
+
+def decide(lib, **kw):
+    a = dict(logits=P, N=8, V=32, n_seq=2, d_in=None, d_out=None, draft_ok=None, tau=0.8, budget=2, remask_budget=3,
+             mask_id=31, min_one=1, pos0=0, max_seeds=4, tok=P, flags=P, remask_cnt=P, maxprob=P, entropy=P,
+             argmax=P, score=P, seed_idx=P, n_seeds=P, stats=None, workspace=P)
+    a.update(kw)
+    return lib.cover_score_decide_fwd(*a.values(), None)
+
+
+@pytest.mark.parametrize("kw", [
+    dict(logits=None), dict(tok=None), dict(flags=None), dict(remask_cnt=None), dict(n_seeds=None),
+    dict(workspace=None), dict(N=0), dict(V=0), dict(n_seq=3), dict(N=8194, n_seq=2), dict(budget=-1),
+    dict(remask_budget=-1), dict(max_seeds=-1), dict(seed_idx=None), dict(logits=P + 2), dict(workspace=P + 4),
+    dict(tok=P + 2),
+])
+def test_decide_invalid_args(lib, kw):
+    assert decide(lib, **kw) == -1
+
+
+def test_decide_workspace_bytes(lib):
+    assert lib.cover_decide_workspace_bytes(8, 2) == 16 + 64
+    assert lib.cover_decide_workspace_bytes(4096, 5) == 32 + 8 * 4096
+    assert lib.cover_decide_workspace_bytes(0, 1) == 0
