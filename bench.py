@@ -13,6 +13,8 @@ Printed JSON line (rank 0):
                memory and its results copied back inside the timed region
   roofline     the attention kernel alone, against the measured bf16 peak
   overhead_vs_no_seed, long_context, scoring: secondary figures
+  decide       scoring fused with one step's decisions (drafting, revision,
+               adaptive seed selection) against scoring + top-k alone
   cpu_baseline the fp64 oracle on a bounded sample of the same workload
 
 ``--impl reference`` times the fp64 oracle (the only reference there is: the
@@ -50,7 +52,7 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-secondary", action="store_true")
-    ap.add_argument("--only", choices=["attn", "score"], default=None,
+    ap.add_argument("--only", choices=["attn", "score", "decide"], default=None,
                     help="time one kernel alone on the workload (for profiler captures)")
     return ap.parse_args()
 
@@ -368,6 +370,8 @@ def run_ours(args):
                                   "frac_of_peak": round(per[LONG_WORKLOAD]["tflops_seeded"] / peak, 4),
                                   "peak_source": roofline["peak_source"]}
         result["scoring_gbs"] = scoring_all
+        result["decide"] = {name: decide_timing(api, torch, W.WORKLOADS[name])
+                            for name in (WORKLOAD, "dream_gqa_l1024")}
         status = api.cover_device_status()
         if status != 0:
             raise RuntimeError(f"device status {api.cover_status_str(status)} in the secondary runs")
@@ -396,6 +400,57 @@ def score_gbs(api, torch, si, iters=20):
         ts.append(a.elapsed_time(b))
     nbytes = si.N * si.V * 2 + si.N * 20 + si.n_seq * si.topk * 8
     return round(nbytes / (statistics.median(ts) * 1e-3) / 1e9, 1)
+
+
+def decide_timing(api, torch, wl, iters=20):
+    """Scoring fused with the decision step vs. scoring + top-k alone, on the same logits.
+
+    Decision parameters follow the paper's setting (tau 0.9, budget B = 15,
+    ReMask budget 5); the decoding state is restored before every call, outside
+    the timed region. GB/s counts the logits read once plus the per-row state.
+    """
+    di = wl.decide_inputs()
+    per = di.N // di.n_seq
+    logits = bf16_dev(di.logits, torch)
+    tok0 = torch.from_numpy(di.tok).cuda()
+    flags0 = torch.from_numpy(di.flags).cuda()
+    rc0 = torch.from_numpy(di.remask_cnt).cuda()
+    tok, flags, rc = tok0.clone(), flags0.clone(), rc0.clone()
+    kw = dict(tau_draft=0.9, draft_budget=15, remask_budget=5, mask_id=di.mask_id, pos0=wl.L - per,
+              max_seeds=wl.score_topk, d_in=torch.from_numpy(di.d_in).cuda(), d_out=torch.from_numpy(di.d_out).cuda(),
+              draft_ok=torch.from_numpy(di.draft_ok).cuda())
+    ws = api.decide_workspace(di.N, di.n_seq)
+    out = api.cover_score_decide_fwd(logits, di.n_seq, tok, flags, rc, workspace=ws, **kw)
+    wsp = api.score_workspace(di.n_seq)
+    sout = api.cover_score_fwd(logits, di.n_seq, wl.score_topk, workspace=wsp)
+    stream = torch.cuda.current_stream()
+
+    def timed(fused):
+        ts = []
+        for _ in range(iters):
+            tok.copy_(tok0)
+            flags.copy_(flags0)
+            rc.copy_(rc0)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            if fused:
+                api.cover_score_decide_fwd(logits, di.n_seq, tok, flags, rc, workspace=ws, out=out, **kw)
+            else:
+                api.cover_score_fwd(logits, di.n_seq, wl.score_topk, workspace=wsp, out=sout)
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        return statistics.median(ts)
+
+    t_dec, t_score = timed(True), timed(False)
+    t_dec, t_score = min(t_dec, timed(True)), min(t_score, timed(False))
+    stats = out["stats"].cpu().numpy()
+    nbytes = di.N * di.V * 2 + di.N * (20 + 12) + di.n_seq * wl.score_topk * 4
+    return {"ms_decide": round(t_dec, 4), "ms_score_topk": round(t_score, 4),
+            "overhead": round((t_dec - t_score) / t_score, 4),
+            "gbs": round(nbytes / (t_dec * 1e-3) / 1e9, 1),
+            "drafted_per_seq": round(float(stats[:, 0].mean()), 2),
+            "seeds_per_seq": round(float(out["n_seeds"].float().mean().item()), 2)}
 
 
 def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, iters=20):
@@ -550,11 +605,19 @@ def run_only(args):
         seeds = torch.from_numpy(ai.seed_idx).cuda()
         out, lse = torch.empty_like(q), torch.empty((wl.B, wl.Hq, wl.L), device="cuda")
         fn = lambda: api.cover_attn_fwd(q, kc, vc, km, vm, seeds, out=out, lse=lse)  # noqa: E731
-    else:
+    elif args.only == "score":
         si = wl.score_inputs()
         logits = bf16_dev(si.logits, torch)
         wsp = api.score_workspace(si.n_seq)
         fn = lambda: api.cover_score_fwd(logits, si.n_seq, si.topk, workspace=wsp)  # noqa: E731
+    else:
+        di = wl.decide_inputs()
+        logits = bf16_dev(di.logits, torch)
+        tok, flags, rc = (torch.from_numpy(x).cuda() for x in (di.tok, di.flags, di.remask_cnt))
+        ws = api.decide_workspace(di.N, di.n_seq)
+        fn = lambda: api.cover_score_decide_fwd(  # noqa: E731
+            logits, di.n_seq, tok, flags, rc, tau_draft=0.9, draft_budget=15, remask_budget=5, mask_id=di.mask_id,
+            pos0=wl.L - di.N // di.n_seq, max_seeds=wl.score_topk, workspace=ws)
     for _ in range(max(args.warmup, 1)):
         fn()
     torch.cuda.synchronize()

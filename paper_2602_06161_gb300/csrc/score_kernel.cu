@@ -54,6 +54,7 @@ constexpr int kChunkBytes = kChunkElems * 2;
 constexpr int kRingStages = 3;
 constexpr int kVecPerThread = kChunkElems / 8 / (kConsumerWarps * 32);   // 4
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kRoundsMax = 32;             // decision step: selections up to this size by rounds
 
 struct RowAcc {
   float m;     // running maximum logit of this thread's elements
@@ -302,53 +303,104 @@ __device__ __forceinline__ int rank_key_row(uint64_t key) {
   return static_cast<int>(0xffffffffu - static_cast<uint32_t>(key));
 }
 
+// The k largest of the n keys in shared memory (keys are distinct, 0 = none),
+// in descending order, by k rounds of a CTA-wide maximum below the previous
+// round's: one barrier per round, the keys untouched. out[t] gets round t's
+// key (0 once the nonzero keys run out). All threads call it with the same k.
+__device__ __forceinline__ void top_rounds(const uint64_t* keys, int n, int k, uint64_t* out,
+                                           unsigned long long (*scratch)[32]) {
+  const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5, nw = nt >> 5;
+  uint64_t prev = ~0ull;
+  for (int t = 0; t < k; ++t) {
+    uint64_t m = 0;
+    for (int i = tid; i < n; i += nt) {
+      const uint64_t x = keys[i];
+      if (x < prev && x > m) m = x;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const uint64_t y = __shfl_xor_sync(0xffffffffu, m, o);
+      m = y > m ? y : m;
+    }
+    if (lane == 0) scratch[t & 1][warp] = m;
+    __syncthreads();
+    m = 0;
+    for (int w = 0; w < nw; ++w) m = scratch[t & 1][w] > m ? scratch[t & 1][w] : m;
+    if (tid == 0) out[t] = m;
+    prev = m;
+    if (m == 0) {
+      for (int r = t + 1 + tid; r < k; r += nt) out[r] = 0;
+      break;
+    }
+  }
+  __syncthreads();
+}
+
 // The last CTA of a segment: one decoding step's decisions for that sequence.
-// Rows written by other CTAs are read through L2 (__ldcg).
+// Rows written by other CTAs are read through L2 (__ldcg). The drafting sort
+// runs only when more rows pass the threshold than the budget allows; the
+// selection sort only when seeds are to be chosen.
 __device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n, const ScoreParams& P) {
   __shared__ unsigned long long s_fallback;
   __shared__ int s_ri[32];
+  __shared__ int s_cnt[4][32];
   __shared__ double s_rd[32];
+  __shared__ unsigned long long s_top[2][32];
+  __shared__ uint64_t s_sel[kRoundsMax];
   __threadfence();
   const DecideArgs& d = P.dec;
-  const int tid = threadIdx.x, nt = blockDim.x;
+  float* sscore = reinterpret_cast<float*>(keys + sort_n);   // per-row seed score
+  const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5, nw = nt >> 5;
   const int base = seg * per_seq;
   if (tid == 0) s_fallback = ~0ull;
   __syncthreads();
 
   // Section 5.2 drafting: masked rows in the allowed set whose confidence exceeds tau
   int ncand = 0;
-  for (int i = tid; i < sort_n; i += nt) {
-    uint64_t key = 0;
-    if (i < per_seq) {
-      const int n = base + i;
-      if (d.tok[n] == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0)) {
-        const float c = __ldcg(P.maxprob + n);
-        if (c > d.tau) {
-          key = rank_key(c, i);
-          ++ncand;
-        }
-        if (d.min_one) {
-          // lowest entropy, then lowest index
-          const uint64_t fb = (static_cast<uint64_t>(order_key(__ldcg(P.entropy + n))) << 32) | static_cast<uint32_t>(i);
-          atomicMin(&s_fallback, static_cast<unsigned long long>(fb));
-        }
+  for (int i = tid; i < per_seq; i += nt) {
+    const int n = base + i;
+    if (d.tok[n] == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0)) {
+      if (__ldcg(P.maxprob + n) > d.tau) ++ncand;
+      if (d.min_one) {
+        // lowest entropy, then lowest index
+        const uint64_t fb = (static_cast<uint64_t>(order_key(__ldcg(P.entropy + n))) << 32) | static_cast<uint32_t>(i);
+        atomicMin(&s_fallback, static_cast<unsigned long long>(fb));
       }
     }
-    keys[i] = key;
   }
   ncand = block_sum(ncand, s_ri);
-  bitonic_sort_desc(keys, sort_n);
+  const bool all_cand = ncand <= d.budget;   // every row above tau is drafted
   int n_drafted = min(ncand, d.budget);
   const bool fallback = n_drafted == 0 && d.min_one && s_fallback != ~0ull;
-  for (int t = tid; t < (fallback ? 1 : n_drafted); t += nt) {
-    const int n = base + (fallback ? static_cast<int>(static_cast<uint32_t>(s_fallback)) : rank_key_row(keys[t]));
-    // a drafted row takes its greedy token, whose uncertainty is ln Z
-    d.tok[n] = __ldcg(P.argmax + n);
-    d.ws_u[n] = __ldcg(d.ws_lnz + n);
-    d.flags[n] = static_cast<uint8_t>(d.flags[n] & ~1u);
+  if (!all_cand) {
+    // more candidates than the budget: the `budget` most confident (ties to the lower index)
+    for (int i = tid; i < sort_n; i += nt) {
+      uint64_t key = 0;
+      if (i < per_seq) {
+        const int n = base + i;
+        const float c = __ldcg(P.maxprob + n);
+        if (d.tok[n] == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0) && c > d.tau) key = rank_key(c, i);
+      }
+      keys[i] = key;
+    }
+    __syncthreads();
+    if (n_drafted <= kRoundsMax)
+      top_rounds(keys, sort_n, n_drafted, s_sel, s_top);
+    else
+      bitonic_sort_desc(keys, sort_n);
+  }
+  if (!all_cand || fallback) {
+    const uint64_t* picked = n_drafted <= kRoundsMax ? s_sel : keys;
+    for (int t = tid; t < (fallback ? 1 : n_drafted); t += nt) {
+      const int n = base + (fallback ? static_cast<int>(static_cast<uint32_t>(s_fallback)) : rank_key_row(picked[t]));
+      // a drafted row takes its greedy token, whose uncertainty is ln Z
+      d.tok[n] = __ldcg(P.argmax + n);
+      d.ws_u[n] = __ldcg(d.ws_lnz + n);
+      d.flags[n] = static_cast<uint8_t>(d.flags[n] & ~1u);
+    }
+    __syncthreads();
   }
   if (fallback) n_drafted = 1;
-  __syncthreads();
 
   // Section 5.2 revision of the previous seeds, Section 3 state update, Section 5.3 seed score
   int kept = 0, replaced = 0, remasked = 0, n_t = 0;
@@ -358,10 +410,20 @@ __device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n,
     if (i < per_seq) {
       const int n = base + i;
       int y = d.tok[n];
-      const uint8_t fl = d.flags[n];
+      uint8_t fl = d.flags[n];
       int rc = d.remask_cnt[n];
+      float u;
+      if (all_cand && y == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0) &&
+          __ldcg(P.maxprob + n) > d.tau) {
+        // drafted (every candidate fits the budget)
+        y = __ldcg(P.argmax + n);
+        u = __ldcg(d.ws_lnz + n);
+        fl = static_cast<uint8_t>(fl & ~1u);
+        d.tok[n] = y;
+      } else {
+        u = __ldcg(d.ws_u + n);
+      }
       const bool was_seed = (fl & 1u) != 0 && y != d.mask_id;
-      float u = __ldcg(d.ws_u + n);
       if (was_seed) {
         const int yh = __ldcg(P.argmax + n);
         if (yh == y) {
@@ -392,19 +454,41 @@ __device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n,
         }
       }
       P.score[n] = s;
+      sscore[i] = s;
     }
     keys[i] = key;
   }
-  kept = block_sum(kept, s_ri);
-  replaced = block_sum(replaced, s_ri);
-  remasked = block_sum(remasked, s_ri);
-  n_t = block_sum(n_t, s_ri);
-  total = block_sum(total, s_rd);
+  // one reduction for the four counts and the score sum
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    kept += __shfl_xor_sync(0xffffffffu, kept, o);
+    replaced += __shfl_xor_sync(0xffffffffu, replaced, o);
+    remasked += __shfl_xor_sync(0xffffffffu, remasked, o);
+    n_t += __shfl_xor_sync(0xffffffffu, n_t, o);
+    total += __shfl_xor_sync(0xffffffffu, total, o);
+  }
+  if (lane == 0) {
+    s_cnt[0][warp] = kept;
+    s_cnt[1][warp] = replaced;
+    s_cnt[2][warp] = remasked;
+    s_cnt[3][warp] = n_t;
+    s_rd[warp] = total;
+  }
+  __syncthreads();
+  kept = replaced = remasked = n_t = 0;
+  total = 0.0;
+  for (int w = 0; w < nw; ++w) {
+    kept += s_cnt[0][w];
+    replaced += s_cnt[1][w];
+    remasked += s_cnt[2][w];
+    n_t += s_cnt[3][w];
+    total += s_rd[w];
+  }
 
   // Section 5.3 adaptive revision rate: n_t pi_t = #{ s_j > mean } = #{ n_t s_j > sum s }
   int above = 0;
   for (int i = tid; i < per_seq; i += nt) {
-    const float s = __ldcg(P.score + base + i);
+    const float s = sscore[i];
     if (s != -INFINITY && static_cast<double>(n_t) * static_cast<double>(s) > total) ++above;
   }
   above = block_sum(above, s_ri);
@@ -413,12 +497,18 @@ __device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n,
   k = min(k, d.max_seeds);
 
   // selection: the k best eligible rows (keys written above)
-  bitonic_sort_desc(keys, sort_n);
+  const uint64_t* best = keys;
+  if (k > 0 && k <= kRoundsMax) {
+    top_rounds(keys, sort_n, k, s_sel, s_top);
+    best = s_sel;
+  } else if (k > 0) {
+    bitonic_sort_desc(keys, sort_n);
+  }
   int chosen = 0;
   for (int t = tid; t < d.max_seeds; t += nt) {
     int pos = -1;
-    if (t < k && t < sort_n && keys[t] != 0) {
-      const int i = rank_key_row(keys[t]);
+    if (t < k && t < sort_n && best[t] != 0) {
+      const int i = rank_key_row(best[t]);
       pos = d.pos0 + i;
       d.flags[base + i] = static_cast<uint8_t>(d.flags[base + i] | 1u);
       ++chosen;
@@ -680,7 +770,9 @@ int launch_score_impl(const ScoreArgs& a, const DecideArgs* d, int* status, cuda
   ScoreParams P{static_cast<const uint16_t*>(a.logits), a.V, per, a.cur_tok, a.d_in, a.d_out, a.eligible,
                 a.topk, sort_n, a.maxprob, a.entropy, a.argmax, a.score, a.topk_idx, a.topk_score, a.counters,
                 d != nullptr ? 1 : 0, d != nullptr ? *d : DecideArgs{}};
-  const size_t keys_bytes = (a.topk > 0 || d != nullptr) ? sizeof(uint64_t) * static_cast<size_t>(sort_n) : 0;
+  // top-k keys; the decision step also keeps a float score per row behind them
+  const size_t keys_bytes = d != nullptr ? (sizeof(uint64_t) + sizeof(float)) * static_cast<size_t>(sort_n)
+                            : a.topk > 0 ? sizeof(uint64_t) * static_cast<size_t>(sort_n) : 0;
   const bool aligned_rows = (a.V % 8) == 0 && (reinterpret_cast<uintptr_t>(a.logits) % 16) == 0;
   if (aligned_rows) {
     const size_t smem = std::max(keys_bytes, static_cast<size_t>(kRingStages) * kChunkBytes);
