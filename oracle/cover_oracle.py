@@ -23,6 +23,9 @@ Everything here is written from the paper's definitions:
   Keep / Replace / ReMask revision of the previous seeds, the state update;
   §5.3: the seed score on the updated state, the adaptive revision rate
   |S_t| = ceil(sqrt(n_t pi_t)) and the exclusions from seed selection.
+* §5.1 (seed K/V cache): the states of the new seeds cached at selection and
+  written over the seed columns of the next step's memory, the masked-input
+  states moving into the diagonal side buffer.
 
 Readings of points the paper leaves open (numbered as in the design notes):
 the cached inputs already hold the overridden memory K', V' (R1); the masked
@@ -444,3 +447,69 @@ def decide_step(conf, yhat, ent, u_cur, u_top, d_in, d_out, tok, flags, remask_c
                                     pick(d_out), pick(tok), pick(flags), pick(remask_cnt), pick(draft_ok),
                                     **params))
     return outs
+
+
+# ----------------------------------------------------------------------------
+# Seed K/V cache (§5.1 "KV cache override yields a stable drafting view"):
+# at selection the per-layer key / value states of the new seeds are cached;
+# at the next step the memory is overridden at the seed positions with them,
+# while the states computed from the masked input at those positions become
+# the diagonal pairs (k_i, v_i) of the leave-one-out views.
+# ----------------------------------------------------------------------------
+
+def _seed_slots(seed_idx, L: int):
+    """Per batch row, the (slot, position) pairs that name a position: in range and
+    not repeating an earlier slot's position (the lowest slot wins, as in R7)."""
+    out = []
+    for b in range(seed_idx.shape[0]):
+        seen, pairs = set(), []
+        for s in range(seed_idx.shape[1]):
+            j = int(seed_idx[b, s])
+            if 0 <= j < L and j not in seen:
+                seen.add(j)
+                pairs.append((s, j))
+        out.append(pairs)
+    return out
+
+
+def seed_kv_gather(k, v, seed_idx):
+    """Cache at selection: cache[b, h, s] = state[b, h, seed_idx[b, s]] for k and v.
+
+    k, v: [B, Hkv, L, D] (any dtype; values are copied, never computed).
+    A slot whose position is out of [0, L) holds zeros; a repeated position is
+    cached again in every slot that names it.
+    """
+    B, H, L, D = k.shape
+    S = seed_idx.shape[1]
+    kc = np.zeros((B, H, S, D), dtype=k.dtype)
+    vc = np.zeros((B, H, S, D), dtype=v.dtype)
+    for b in range(B):
+        for s in range(S):
+            j = int(seed_idx[b, s])
+            if 0 <= j < L:
+                kc[b, :, s] = k[b, :, j]
+                vc[b, :, s] = v[b, :, j]
+    return kc, vc
+
+
+def seed_kv_override(k, v, seed_idx, k_cache, v_cache):
+    """Override at the next step.
+
+    k, v: the layer's states from the masked input, [B, Hkv, L, D];
+    k_cache, v_cache: the states cached at selection, [B, Hkv, S, D].
+    Returns (k', v', k_mask, v_mask): k'/v' equal k/v except that row j of
+    every seed (b, s, j) holds the cached row s; k_mask/v_mask row s holds the
+    masked-input state at j (the pair (k_j, v_j) restored on the diagonal).
+    Slots that do not name a position (out of range, or a position already
+    named by a lower slot) keep their cache row and change no memory row.
+    """
+    L = k.shape[2]
+    k2, v2 = k.copy(), v.copy()
+    km, vm = k_cache.copy(), v_cache.copy()
+    for b, pairs in enumerate(_seed_slots(seed_idx, L)):
+        for s, j in pairs:
+            k2[b, :, j] = k_cache[b, :, s]
+            v2[b, :, j] = v_cache[b, :, s]
+            km[b, :, s] = k[b, :, j]
+            vm[b, :, s] = v[b, :, j]
+    return k2, v2, km, vm
