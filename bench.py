@@ -15,6 +15,7 @@ Printed JSON line (rank 0):
   overhead_vs_no_seed, long_context, scoring: secondary figures
   decide       scoring fused with one step's decisions (drafting, revision,
                adaptive seed selection) against scoring + top-k alone
+  seed_kv      per-layer seed K/V cache gather and override swap
   cpu_baseline the fp64 oracle on a bounded sample of the same workload
 
 ``--impl reference`` times the fp64 oracle (the only reference there is: the
@@ -347,6 +348,7 @@ def run_ours(args):
     # ---------------- secondary: every named workload ----------------
     if not args.no_secondary:
         per = {WORKLOAD: seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops)}
+        kv_all = {WORKLOAD: kv_timing(api, torch, kc, vc, seeds)}
         del q, kc, vc, km, vm, logits
         torch.cuda.empty_cache()
         scoring_all = {WORKLOAD: scoring["gbs"]}
@@ -359,6 +361,7 @@ def run_ours(args):
             oout = torch.empty_like(oq)
             olse = torch.empty((ow.B, ow.Hq, ow.L), dtype=torch.float32, device="cuda")
             per[name] = seed_overhead(api, torch, oq, okc, ovc, okm, ovm, oseeds, oout, olse, ow.attn_flops)
+            kv_all[name] = kv_timing(api, torch, okc, ovc, oseeds)
             del oq, okc, ovc, okm, ovm, oseeds, oout, olse
             osi = ow.score_inputs()
             if osi is not None:
@@ -370,6 +373,7 @@ def run_ours(args):
                                   "frac_of_peak": round(per[LONG_WORKLOAD]["tflops_seeded"] / peak, 4),
                                   "peak_source": roofline["peak_source"]}
         result["scoring_gbs"] = scoring_all
+        result["seed_kv"] = kv_all
         result["decide"] = {name: decide_timing(api, torch, W.WORKLOADS[name])
                             for name in (WORKLOAD, "dream_gqa_l1024")}
         status = api.cover_device_status()
@@ -451,6 +455,40 @@ def decide_timing(api, torch, wl, iters=20):
             "gbs": round(nbytes / (t_dec * 1e-3) / 1e9, 1),
             "drafted_per_seq": round(float(stats[:, 0].mean()), 2),
             "seeds_per_seq": round(float(out["n_seeds"].float().mean().item()), 2)}
+
+
+def kv_timing(api, torch, k, v, seeds, iters=20):
+    """Per-layer seed K/V cache traffic: gather at selection, override swap at the next step.
+
+    Times each call alone (median of `iters`); GB/s counts the bytes each call
+    moves (gather: read the seed rows, write the cache; override: read and
+    write both the seed rows and the cache rows, for k and v).
+    """
+    B, Hkv, L, D = k.shape
+    S = seeds.shape[1]
+    stream = torch.cuda.current_stream()
+    kc, vc = api.cover_seed_kv_gather(k, v, seeds)
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        ts = []
+        for _ in range(iters):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        return statistics.median(ts)
+
+    t_g = timed(lambda: api.cover_seed_kv_gather(k, v, seeds, k_cache=kc, v_cache=vc))
+    t_o = timed(lambda: api.cover_seed_kv_override(k, v, seeds, kc, vc))   # an even count leaves k, v as they were
+    row = D * k.element_size()
+    g_bytes = 4 * B * Hkv * S * row
+    return {"ms_gather": round(t_g, 4), "ms_override": round(t_o, 4),
+            "gbs_gather": round(g_bytes / (t_g * 1e-3) / 1e9, 1),
+            "gbs_override": round(2 * g_bytes / (t_o * 1e-3) / 1e9, 1)}
 
 
 def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, iters=20):

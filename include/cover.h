@@ -168,6 +168,41 @@ int cover_score_fwd_noalloc(const void* logits, int N, int V, int n_seq,
                             int32_t* topk_idx, float* topk_score, void* stream);
 
 /*
+ * Seed key/value cache (Section 5.1, "KV cache override yields a stable
+ * drafting view"), per layer. k, v: the layer's states [B, Hkv, L, D];
+ * k_cache, v_cache: [B, Hkv, n_seeds, D]; seed_idx: int32 [B, n_seeds]
+ * positions (the row of the previous step's cover_score_decide_fwd output
+ * works as is). Elements are elem_bytes (2 for bf16, 4 for fp32) bytes; a row
+ * (D * elem_bytes) must be a multiple of 16 bytes and every pointer 16-byte
+ * aligned. All pointers are device pointers owned by the caller.
+ *
+ * A slot names its position when the position is in [0, L) and no lower slot
+ * of the same batch row names it (the lowest slot wins, as in cover_attn_fwd).
+ *
+ * cover_seed_kv_gather (at selection, step t-1): k_cache[b, h, s] =
+ *   k[b, h, seed_idx[b, s]], likewise v; a slot with an out-of-range position
+ *   gets zeros (a repeated position is copied again).
+ * cover_seed_kv_override (at step t, after the layer's k, v were computed from
+ *   the input with the seeds masked): swaps row seed_idx[b, s] of k / v with
+ *   row s of k_cache / v_cache for every slot that names a position. Afterwards
+ *   k, v hold the overridden memory K', V' and k_cache, v_cache hold the
+ *   masked-input pairs (k_i, v_i): exactly cover_attn_fwd's k_cached,
+ *   v_cached, k_seedmask, v_seedmask. Slots that name no position leave both
+ *   buffers untouched.
+ * n_seeds = 0 is a no-op (seed pointers may then be NULL).
+ * Errors: COVER_ERR_INVALID_ARG for a NULL required pointer, B, Hkv, L or D
+ * < 1, n_seeds < 0, elem_bytes not 2 or 4, a row that is not a multiple of 16
+ * bytes or is longer than 64 KB, or a misaligned pointer; COVER_ERR_UNSUPPORTED if B * Hkv > 2^31 - 1 or
+ * n_seeds > 1048560; COVER_ERR_CUDA for a launch failure.
+ */
+int cover_seed_kv_gather(const void* k, const void* v, const int32_t* seed_idx, int n_seeds,
+                         int B, int Hkv, int L, int D, int elem_bytes,
+                         void* k_cache, void* v_cache, void* stream);
+int cover_seed_kv_override(void* k, void* v, const int32_t* seed_idx, int n_seeds,
+                           int B, int Hkv, int L, int D, int elem_bytes,
+                           void* k_cache, void* v_cache, void* stream);
+
+/*
  * One decoding step's decisions, fused behind the scoring pass
  * (Section 5.2 "Threshold drafting" and the Keep / Replace / ReMask revision
  * rule, Section 3 state update, Section 5.3 stability-aware seed score,

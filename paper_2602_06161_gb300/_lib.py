@@ -24,6 +24,8 @@ _SIGNATURES = {
     "cover_score_workspace_bytes": (ctypes.c_size_t, [_I]),
     "cover_score_fwd": (_I, [_P, _I, _I, _I, _P, _P, _P, _P, _I, _P, _P, _P, _P, _P, _P, _P, _P]),
     "cover_score_fwd_noalloc": (_I, [_P, _I, _I, _I, _P, _P, _P, _P, _I, _P, _P, _P, _P, _P, _P, _P]),
+    "cover_seed_kv_gather": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
+    "cover_seed_kv_override": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
     "cover_decide_workspace_bytes": (ctypes.c_size_t, [_I, _I]),
     "cover_score_decide_fwd": (_I, [_P, _I, _I, _I, _P, _P, _P, ctypes.c_float, _I, _I, _I, _I, _I, _I,
                                     _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P]),

@@ -186,6 +186,45 @@ def cover_score_fwd_noalloc(logits, n_seq: int, topk: int, *, cur_tok=None, d_in
     return out
 
 
+def _seed_kv(fn_name, k, v, seed_idx, k_cache, v_cache, stream):
+    if k.dtype not in (torch.bfloat16, torch.float32):
+        raise TypeError("k must be bfloat16 or float32")
+    _need(k, "k", k.dtype, 4)
+    _need(v, "v", k.dtype, 4)
+    B, Hkv, L, D = k.shape
+    if tuple(v.shape) != (B, Hkv, L, D):
+        raise ValueError("v must match k")
+    S = 0 if seed_idx is None else int(seed_idx.shape[1])
+    if S > 0:
+        _need(seed_idx, "seed_idx", torch.int32, 2)
+        if tuple(seed_idx.shape) != (B, S):
+            raise ValueError("seed_idx must be [B, S]")
+        if k_cache is None:
+            k_cache = torch.empty((B, Hkv, S, D), dtype=k.dtype, device=k.device)
+            v_cache = torch.empty_like(k_cache)
+        _need(k_cache, "k_cache", k.dtype, 4)
+        _need(v_cache, "v_cache", k.dtype, 4)
+        if tuple(k_cache.shape) != (B, Hkv, S, D) or tuple(v_cache.shape) != (B, Hkv, S, D):
+            raise ValueError("k_cache / v_cache must be [B, Hkv, S, D]")
+    code = getattr(_lib.load(), fn_name)(
+        _ptr(k), _ptr(v), _ptr(seed_idx) if S else None, S, B, Hkv, L, D, k.element_size(),
+        _ptr(k_cache) if S else None, _ptr(v_cache) if S else None, _stream(stream))
+    _lib.check(fn_name, code)
+    return k_cache, v_cache
+
+
+def cover_seed_kv_gather(k, v, seed_idx, *, k_cache=None, v_cache=None, stream=None):
+    """Cache the seeds' states at selection: returns (k_cache, v_cache) [B, Hkv, S, D]."""
+    return _seed_kv("cover_seed_kv_gather", k, v, seed_idx, k_cache, v_cache, stream)
+
+
+def cover_seed_kv_override(k, v, seed_idx, k_cache, v_cache, *, stream=None):
+    """Swap the cached seed states into k, v (in place); the caches then hold the masked-input pairs."""
+    if seed_idx is not None and seed_idx.shape[1] > 0 and (k_cache is None or v_cache is None):
+        raise ValueError("k_cache and v_cache are required")
+    return _seed_kv("cover_seed_kv_override", k, v, seed_idx, k_cache, v_cache, stream)
+
+
 def cover_decide_workspace_bytes(N: int, n_seq: int) -> int:
     return int(_lib.load().cover_decide_workspace_bytes(int(N), int(n_seq)))
 

@@ -134,6 +134,34 @@ int cover_score_fwd_noalloc(const void* logits, int N, int V, int n_seq, const i
   return cover::launch_score_noalloc(a, st, static_cast<cudaStream_t>(stream));
 }
 
+static int seed_kv_call(bool swap, void* k, void* v, const int32_t* seed_idx, int n_seeds, int B, int Hkv, int L,
+                        int D, int elem_bytes, void* k_cache, void* v_cache, void* stream) {
+  if (k == nullptr || v == nullptr) return COVER_ERR_INVALID_ARG;
+  if (B < 1 || Hkv < 1 || L < 1 || D < 1 || n_seeds < 0) return COVER_ERR_INVALID_ARG;
+  if (elem_bytes != 2 && elem_bytes != 4) return COVER_ERR_INVALID_ARG;
+  const long long row = static_cast<long long>(D) * elem_bytes;
+  if (row % 16 != 0 || row > 65536) return COVER_ERR_INVALID_ARG;
+  if (n_seeds > 0 && (seed_idx == nullptr || k_cache == nullptr || v_cache == nullptr)) return COVER_ERR_INVALID_ARG;
+  if (!aligned(k, 16) || !aligned(v, 16)) return COVER_ERR_INVALID_ARG;
+  if (n_seeds > 0 && (!aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(seed_idx, 4)))
+    return COVER_ERR_INVALID_ARG;
+  if (n_seeds == 0) return COVER_OK;
+  const int rc = cover::launch_seed_kv(swap, k, v, seed_idx, n_seeds, B, Hkv, L, static_cast<int>(row), k_cache,
+                                       v_cache, static_cast<cudaStream_t>(stream));
+  return rc == -2 ? COVER_ERR_UNSUPPORTED : rc == 0 ? COVER_OK : COVER_ERR_CUDA;
+}
+
+int cover_seed_kv_gather(const void* k, const void* v, const int32_t* seed_idx, int n_seeds, int B, int Hkv, int L,
+                         int D, int elem_bytes, void* k_cache, void* v_cache, void* stream) {
+  return seed_kv_call(false, const_cast<void*>(k), const_cast<void*>(v), seed_idx, n_seeds, B, Hkv, L, D, elem_bytes,
+                      k_cache, v_cache, stream);
+}
+
+int cover_seed_kv_override(void* k, void* v, const int32_t* seed_idx, int n_seeds, int B, int Hkv, int L, int D,
+                           int elem_bytes, void* k_cache, void* v_cache, void* stream) {
+  return seed_kv_call(true, k, v, seed_idx, n_seeds, B, Hkv, L, D, elem_bytes, k_cache, v_cache, stream);
+}
+
 size_t cover_decide_workspace_bytes(int N, int n_seq) {
   if (N < 1 || n_seq < 1) return 0;
   // per-segment counters, then u and ln Z per row

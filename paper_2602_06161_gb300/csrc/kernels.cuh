@@ -75,6 +75,11 @@ int launch_score_decide(const ScoreArgs& a, const DecideArgs& d, int* status, cu
 constexpr int kNoAllocMaxSegments = 4096;
 int launch_score_noalloc(ScoreArgs a, int* status, cudaStream_t stream);
 
+// Seed K/V cache (Section 5.1): gather (override_swap = false) or the override
+// swap (true) of rows of row_bytes (a multiple of 16) bytes.
+int launch_seed_kv(bool override_swap, void* k, void* v, const int32_t* seed_idx, int n_seeds, int B, int Hkv, int L,
+                   int row_bytes, void* k_cache, void* v_cache, cudaStream_t stream);
+
 int launch_umma_tile(const void* a, const void* b, const void* p, const void* v, float* c1, float* c2, int* status,
                      cudaStream_t stream);
 int launch_wait_timeout(uint64_t limit_ns, int* status, cudaStream_t stream);

@@ -124,3 +124,21 @@ def test_decide_workspace_bytes(lib):
     assert lib.cover_decide_workspace_bytes(8, 2) == 16 + 64
     assert lib.cover_decide_workspace_bytes(4096, 5) == 32 + 8 * 4096
     assert lib.cover_decide_workspace_bytes(0, 1) == 0
+
+
+@pytest.mark.parametrize("fn", ["cover_seed_kv_gather", "cover_seed_kv_override"])
+@pytest.mark.parametrize("kw", [
+    dict(k=None), dict(v=None), dict(B=0), dict(Hkv=0), dict(L=0), dict(D=0), dict(n_seeds=-1),
+    dict(elem_bytes=1), dict(elem_bytes=8), dict(D=4), dict(D=65536), dict(seed_idx=None), dict(k_cache=None),
+    dict(v_cache=None), dict(k=P + 8), dict(k_cache=P + 8), dict(seed_idx=P + 2),
+])
+def test_seed_kv_invalid_args(lib, fn, kw):
+    a = dict(k=P, v=P, seed_idx=P, n_seeds=4, B=2, Hkv=2, L=16, D=128, elem_bytes=2, k_cache=P, v_cache=P)
+    a.update(kw)
+    assert getattr(lib, fn)(*a.values(), None) == -1
+
+
+def test_seed_kv_no_seeds_is_a_noop(lib):
+    # nothing to move: returns before touching the device
+    assert lib.cover_seed_kv_override(P, P, None, 0, 2, 2, 16, 128, 2, None, None, None) == 0
+    assert lib.cover_seed_kv_gather(P, P, None, 0, 2, 2, 16, 128, 2, None, None, None) == 0
