@@ -469,8 +469,8 @@ def kv_timing(api, torch, k, v, seeds, iters=20):
     stream = torch.cuda.current_stream()
     kc, vc = api.cover_seed_kv_gather(k, v, seeds)
 
-    def timed(fn):
-        for _ in range(3):
+    def timed(fn, warm=4):
+        for _ in range(warm):
             fn()
         ts = []
         for _ in range(iters):
@@ -483,7 +483,7 @@ def kv_timing(api, torch, k, v, seeds, iters=20):
         return statistics.median(ts)
 
     t_g = timed(lambda: api.cover_seed_kv_gather(k, v, seeds, k_cache=kc, v_cache=vc))
-    t_o = timed(lambda: api.cover_seed_kv_override(k, v, seeds, kc, vc))   # an even count leaves k, v as they were
+    t_o = timed(lambda: api.cover_seed_kv_override(k, v, seeds, kc, vc))   # 24 swaps: k, v end as they began
     row = D * k.element_size()
     g_bytes = 4 * B * Hkv * S * row
     return {"ms_gather": round(t_g, 4), "ms_override": round(t_o, 4),
