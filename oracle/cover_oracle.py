@@ -45,7 +45,10 @@ by the caller's seed capacity and the number of eligible positions (R23);
 "selected in the previous step" means S_{t-1} (R24); the seed score uses the
 uncertainty of the updated token, so a drafted or replaced position takes
 -log p(greedy token) (R25); drafting is limited to a caller-given set of
-positions, the active block of semi-autoregressive decoding (R26).
+positions, the active block of semi-autoregressive decoding (R26). With a
+prefix cache (§6.6) only the active block's queries are computed: query row r
+is memory position q0 + r, and a seed outside that window only overrides the
+memory (R27).
 
 Every function is pinned by ``tests/test_oracle_pins.py`` against closed forms,
 hand-worked fixtures, a library routine (torch float64 SDPA) and brute force.
@@ -179,6 +182,34 @@ def override_attention(q, kc, vc, km, vm, seed_idx):
                 s = int(slot[b, i])
                 K, V = view_for_row(Kp, Vp, int(i), (km[b, hkv, s], vm[b, hkv, s]))
                 out[b, hq, i], lse[b, hq, i], _ = attention_row(q[b, hq, i], K, V)
+    return out, lse
+
+
+def override_attention_window(q, kc, vc, km, vm, seed_idx, q0: int):
+    """Two-view attention for a window of query rows (§6.6 prefix cache; reading R27).
+
+    q [B,Hq,Lq,D] holds the queries of memory positions q0 .. q0+Lq-1 (the
+    active block); kc/vc [B,Hkv,Lk,D] are K', V' over every position; seeds are
+    memory positions in [0, Lk). Row r is computed as memory position q0 + r:
+    attention over K', V', or, when that position is a seed, over its
+    leave-one-out view. Seeds outside the window change nothing here.
+    """
+    B, Hq, Lq, D = q.shape
+    Hkv, Lk = kc.shape[1], kc.shape[2]
+    G = Hq // Hkv
+    S = 0 if seed_idx is None else seed_idx.shape[1]
+    slot = route_seeds(seed_idx, Lk)[0] if S else np.full((B, Lk), -1, np.int32)
+    out = np.zeros((B, Hq, Lq, D))
+    lse = np.zeros((B, Hq, Lq))
+    for b in range(B):
+        for hq in range(Hq):
+            hkv = hq // G
+            for r in range(Lq):
+                i = q0 + r
+                s = int(slot[b, i])
+                pair = (km[b, hkv, s], vm[b, hkv, s]) if s >= 0 else None
+                K, V = view_for_row(kc[b, hkv], vc[b, hkv], i, pair)
+                out[b, hq, r], lse[b, hq, r], _ = attention_row(q[b, hq, r], K, V)
     return out, lse
 
 

@@ -423,3 +423,29 @@ def test_planted_entropy_log_base_is_caught(golden_dir, monkeypatch):
     x = G.array(g["logits"])[None, :]
     r = oracle.score_rows(x)
     assert abs(r["entropy"][0] / math.log(2) - G.value(g["entropy"])) > 1e-3
+
+
+# ----------------------------------------------------------------------------
+# Prefix-cache window (Section 6.6): a window of query rows over the full memory
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("q0,Lq", [(0, 24), (5, 7), (13, 11), (23, 1), (0, 1)])
+def test_window_rows_equal_the_square_rows(q0, Lq):
+    # attention rows are independent: the window's rows are the square problem's rows q0 .. q0+Lq-1
+    rng = np.random.default_rng(40 + q0)
+    q, kc, vc, km, vm, seeds = rand_case(2, 4, 2, 24, 8, 6, rng=rng)
+    full, full_lse = oracle.override_attention(q, kc, vc, km, vm, seeds)
+    out, lse = oracle.override_attention_window(q[:, :, q0:q0 + Lq], kc, vc, km, vm, seeds, q0)
+    assert np.max(np.abs(out - full[:, :, q0:q0 + Lq])) < 1e-12
+    assert np.max(np.abs(lse - full_lse[:, :, q0:q0 + Lq])) < 1e-12
+
+
+def test_window_with_seeds_outside_is_plain_attention():
+    # seeds outside the query window only shape the memory: the window rows are textbook
+    # attention over K', V' (torch float64 SDPA)
+    rng = np.random.default_rng(47)
+    q, kc, vc, km, vm, _ = rand_case(1, 2, 1, 20, 8, 3, rng=rng)
+    seeds = np.array([[0, 3, 17]], dtype=np.int32)
+    out, lse = oracle.override_attention_window(q[:, :, 5:15], kc, vc, km, vm, seeds, 5)
+    ref, ref_lse = sdpa_reference(q[:, :, 5:15], kc, vc)
+    assert np.max(np.abs(out - ref)) < 1e-12 and np.max(np.abs(lse - ref_lse)) < 1e-12
