@@ -85,6 +85,30 @@ int cover_attn_fwd_f32(const float* q, const float* k_cached, const float* v_cac
                        float* out, float* lse, void* stream);
 
 /*
+ * Prefix-cache variant (Section 6.6 "Compatibility with Fast-dLLM": only the
+ * active block's queries are recomputed while the memory holds every
+ * position). The memory k_cached / v_cached is [B, Hkv, Lk, D] (overridden at
+ * the seeds, as above); the queries q and the outputs out / lse are
+ * [B, Hq, Lq, D] / [B, Hq, Lq], and query row r sits at memory position
+ * q0 + r (0 <= q0, q0 + Lq <= Lk). seed_idx holds memory positions in
+ * [0, Lk); a seed inside [q0, q0 + Lq) gets its leave-one-out view on the
+ * diagonal column q0 + r, a seed outside the window affects only the memory.
+ * With Lq = Lk and q0 = 0 this is cover_attn_fwd. Types, layouts, ownership
+ * and errors as cover_attn_fwd / cover_attn_fwd_f32, plus
+ * COVER_ERR_INVALID_ARG for Lq < 1, Lk < 1, q0 < 0 or q0 + Lq > Lk.
+ */
+int cover_attn_fwd_prefix(const void* q, const void* k_cached, const void* v_cached,
+                          const void* k_seedmask, const void* v_seedmask,
+                          const int32_t* seed_idx, int n_seeds,
+                          int B, int Hq, int Hkv, int Lq, int Lk, int q0, int D,
+                          void* out, float* lse, void* stream);
+int cover_attn_fwd_prefix_f32(const float* q, const float* k_cached, const float* v_cached,
+                              const float* k_seedmask, const float* v_seedmask,
+                              const int32_t* seed_idx, int n_seeds,
+                              int B, int Hq, int Hkv, int Lq, int Lk, int q0, int D,
+                              float* out, float* lse, void* stream);
+
+/*
  * Seed routing as the attention kernels see it (seed-set semantics of
  * Sections 3 and 5.1), exported for checking.
  *   slot_out   [B, L] int32: slot s of the seed naming position r, else -1

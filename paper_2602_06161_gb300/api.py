@@ -88,6 +88,55 @@ def cover_attn_fwd_f32(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, 
                  out, lse, want_lse, stream)
 
 
+def _attn_prefix(fn_name, dtype, q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, q0, out, lse, want_lse,
+                 stream):
+    _need(q, "q", dtype, 4)
+    _need(k_cached, "k_cached", dtype, 4)
+    _need(v_cached, "v_cached", dtype, 4)
+    B, Hq, Lq, D = q.shape
+    Hkv, Lk = k_cached.shape[1], k_cached.shape[2]
+    if tuple(k_cached.shape) != (B, Hkv, Lk, D) or tuple(v_cached.shape) != (B, Hkv, Lk, D):
+        raise ValueError("k_cached / v_cached must be [B, Hkv, Lk, D] matching q")
+    n_seeds = 0 if seed_idx is None else int(seed_idx.shape[1])
+    if n_seeds > 0:
+        _need(seed_idx, "seed_idx", torch.int32, 2)
+        _need(k_seedmask, "k_seedmask", dtype, 4)
+        _need(v_seedmask, "v_seedmask", dtype, 4)
+        if tuple(seed_idx.shape) != (B, n_seeds):
+            raise ValueError("seed_idx must be [B, S]")
+        if tuple(k_seedmask.shape) != (B, Hkv, n_seeds, D) or tuple(v_seedmask.shape) != (B, Hkv, n_seeds, D):
+            raise ValueError("k_seedmask / v_seedmask must be [B, Hkv, S, D]")
+    if out is None:
+        out = torch.empty_like(q)
+    else:
+        _need(out, "out", dtype, 4)
+    if lse is None and want_lse:
+        lse = torch.empty((B, Hq, Lq), dtype=torch.float32, device=q.device)
+    elif lse is not None:
+        _need(lse, "lse", torch.float32, 3)
+    code = getattr(_lib.load(), fn_name)(
+        _ptr(q), _ptr(k_cached), _ptr(v_cached),
+        _ptr(k_seedmask) if n_seeds else None, _ptr(v_seedmask) if n_seeds else None,
+        _ptr(seed_idx) if n_seeds else None, n_seeds, B, Hq, Hkv, Lq, Lk, int(q0), D,
+        _ptr(out), _ptr(lse), _stream(stream))
+    _lib.check(fn_name, code)
+    return out, lse
+
+
+def cover_attn_fwd_prefix(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, seed_idx=None, *, q0: int,
+                          out=None, lse=None, want_lse=True, stream=None):
+    """Two-view attention for a window of Lq query rows at memory positions q0 .. q0+Lq-1 (bf16)."""
+    return _attn_prefix("cover_attn_fwd_prefix", torch.bfloat16, q, k_cached, v_cached, k_seedmask, v_seedmask,
+                        seed_idx, q0, out, lse, want_lse, stream)
+
+
+def cover_attn_fwd_prefix_f32(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, seed_idx=None, *, q0: int,
+                              out=None, lse=None, want_lse=True, stream=None):
+    """The prefix-window attention in fp32 (CUDA cores)."""
+    return _attn_prefix("cover_attn_fwd_prefix_f32", torch.float32, q, k_cached, v_cached, k_seedmask, v_seedmask,
+                        seed_idx, q0, out, lse, want_lse, stream)
+
+
 def cover_seed_route(seed_idx: Optional[torch.Tensor], B: int, L: int, *, device=None, stream=None):
     """Seed routing as the kernels see it: (slot [B,L] int32, bitmap [B,ceil(L/128),4] int32 bits, n_invalid)."""
     n_seeds = 0 if seed_idx is None else int(seed_idx.shape[1])

@@ -92,7 +92,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ CUtensorMap tm_v, const __nv_bfloat16* __restrict__ k_seedmask,
                      const __nv_bfloat16* __restrict__ v_seedmask, const int32_t* __restrict__ seed_idx, int n_seeds,
-                     int Hq, int Hkv, int L, int n_mblk, float scale_log2, __nv_bfloat16* __restrict__ out,
+                     int Hq, int Hkv, int Lq, int Lk, int q0, int n_mblk, float scale_log2,
+                     __nv_bfloat16* __restrict__ out,
                      float* __restrict__ lse, int* status) {
   extern __shared__ uint8_t smem_raw[];
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -104,8 +105,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int b = blockIdx.x / (n_mblk * Hq);
   const int hkv = hq / (Hq / Hkv);
   const int row0 = mblk * kRowsPerCta;
-  const int nkv = (L + kBN - 1) / kBN;
-  const int tail_valid = L - (nkv - 1) * kBN;   // valid keys in the last KV tile (1..128)
+  const int nkv = (Lk + kBN - 1) / kBN;
+  const int tail_valid = Lk - (nkv - 1) * kBN;   // valid keys in the last KV tile (1..128)
 
   // ---------------- prologue ----------------
   if (tid == 0) {
@@ -133,7 +134,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
-  route_scan(sm.slot, seed_idx + static_cast<size_t>(b) * n_seeds, n_seeds, row0, kRowsPerCta, L, tid, kThreads);
+  // query row r of this CTA sits at memory position q0 + row0 + r
+  route_scan(sm.slot, seed_idx + static_cast<size_t>(b) * n_seeds, n_seeds, q0 + row0, kRowsPerCta, Lk, tid,
+             kThreads);
   __syncthreads();
   const uint32_t tbase = sm.tmem_base;
 
@@ -249,8 +252,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t o_addr = trow + col_o(qt);
     const int grow = row0 + qt * kBM + r;
     const int my_slot = sm.slot[qt * kBM + r];
-    const bool is_seed = my_slot != kNoSlot;
-    const int diag_j = (row0 + qt * kBM) / kBN;
+    const bool is_seed = my_slot != kNoSlot && grow < Lq;
+    // the diagonal of this row: KV tile and column of memory position q0 + grow
+    const int diag_j = (q0 + grow) / kBN;
+    const int diag_c = (q0 + grow) % kBN;
     float m_run = -INFINITY, l_run = 0.0f;
     bool ok = true;
 
@@ -300,11 +305,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < kBN; ++c)
           if (c >= tail_valid) s[c] = -INFINITY;
       }
-      if (j == diag_j && __any_sync(0xffffffffu, is_seed)) {
+      if (__any_sync(0xffffffffu, is_seed && j == diag_j)) {
         // exclusion of the cached diagonal term of a seed row
+        const bool here = is_seed && j == diag_j;
 #pragma unroll
         for (int c = 0; c < kBN; ++c)
-          if (is_seed && c == r) s[c] = -INFINITY;
+          if (here && c == diag_c) s[c] = -INFINITY;
       }
       // row maximum: four independent 3-input max chains
       float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
@@ -395,9 +401,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         m_run = m2;
       }
-      if (grow < L) {
+      if (grow < Lq) {
         const float inv = 1.0f / l_run;
-        uint4* dst = reinterpret_cast<uint4*>(out + ((static_cast<size_t>(b) * Hq + hq) * L + grow) * kD);
+        uint4* dst = reinterpret_cast<uint4*>(out + ((static_cast<size_t>(b) * Hq + hq) * Lq + grow) * kD);
 #pragma unroll
         for (int ch = 0; ch < 16; ++ch) {
           uint4 w;
@@ -408,7 +414,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           dst[ch] = w;
         }
         if (lse != nullptr)
-          lse[(static_cast<size_t>(b) * Hq + hq) * L + grow] = (m_run + log2f(l_run)) * 0.6931471805599453f;
+          lse[(static_cast<size_t>(b) * Hq + hq) * Lq + grow] = (m_run + log2f(l_run)) * 0.6931471805599453f;
       }
     }
   }
@@ -424,11 +430,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) {
   CUtensorMap tq, tk, tv;
-  if (!make_bf16_map_4d(&tq, a.q, kD, a.L, a.Hq, a.B, kBM) ||
+  if (!make_bf16_map_4d(&tq, a.q, kD, a.Lq, a.Hq, a.B, kBM) ||
       !make_bf16_map_4d(&tk, a.k_cached, kD, a.L, a.Hkv, a.B, kBN) ||
       !make_bf16_map_4d(&tv, a.v_cached, kD, a.L, a.Hkv, a.B, kBN))
     return -3;
-  const int n_mblk = (a.L + kRowsPerCta - 1) / kRowsPerCta;
+  const int n_mblk = (a.Lq + kRowsPerCta - 1) / kRowsPerCta;
   const long long grid = static_cast<long long>(n_mblk) * a.Hq * a.B;
   if (grid > 0x7fffffffLL) return -2;
   const size_t smem = sizeof(AttnSmem) + 1024;
@@ -446,7 +452,7 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
   attn_bf16_kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
       tq, tk, tv, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
-      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.L, n_mblk, scale_log2, static_cast<__nv_bfloat16*>(a.out), a.lse,
+      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, scale_log2, static_cast<__nv_bfloat16*>(a.out), a.lse,
       status);
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }

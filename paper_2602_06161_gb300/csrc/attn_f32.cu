@@ -26,15 +26,16 @@ template <int D>
 __global__ void __launch_bounds__(kWarps * 32)
     attn_f32_kernel(const float* __restrict__ q, const float* __restrict__ kc, const float* __restrict__ vc,
                     const float* __restrict__ km, const float* __restrict__ vm, const int32_t* __restrict__ seed_idx,
-                    int n_seeds, int B, int Hq, int Hkv, int L, float* __restrict__ out, float* __restrict__ lse) {
+                    int n_seeds, int B, int Hq, int Hkv, int Lq, int L, int q0, float* __restrict__ out,
+                    float* __restrict__ lse) {
   constexpr int E = D / 32;
   const int lane = threadIdx.x & 31;
   const long long row = static_cast<long long>(blockIdx.x) * kWarps + threadIdx.x / 32;
-  const long long rows = static_cast<long long>(B) * Hq * L;
+  const long long rows = static_cast<long long>(B) * Hq * Lq;
   if (row >= rows) return;
-  const int i = static_cast<int>(row % L);
-  const int hq = static_cast<int>((row / L) % Hq);
-  const int b = static_cast<int>(row / (static_cast<long long>(L) * Hq));
+  const int i = q0 + static_cast<int>(row % Lq);   // memory position of this query row
+  const int hq = static_cast<int>((row / Lq) % Hq);
+  const int b = static_cast<int>(row / (static_cast<long long>(Lq) * Hq));
   const int hkv = hq / (Hq / Hkv);
   const float scale = 1.0f / sqrtf(static_cast<float>(D));
 
@@ -96,7 +97,7 @@ __global__ void __launch_bounds__(kWarps * 32)
 }  // namespace
 
 int launch_attn_f32(const AttnArgs& a, int* /*status*/, cudaStream_t stream) {
-  const long long rows = static_cast<long long>(a.B) * a.Hq * a.L;
+  const long long rows = static_cast<long long>(a.B) * a.Hq * a.Lq;
   const long long blocks = (rows + kWarps - 1) / kWarps;
   if (blocks > 0x7fffffffLL) return -2;
   const float* q = static_cast<const float*>(a.q);
@@ -107,10 +108,10 @@ int launch_attn_f32(const AttnArgs& a, int* /*status*/, cudaStream_t stream) {
   float* out = static_cast<float*>(a.out);
   if (a.D == 64)
     attn_f32_kernel<64><<<static_cast<unsigned>(blocks), kWarps * 32, 0, stream>>>(
-        q, kc, vc, km, vm, a.seed_idx, a.n_seeds, a.B, a.Hq, a.Hkv, a.L, out, a.lse);
+        q, kc, vc, km, vm, a.seed_idx, a.n_seeds, a.B, a.Hq, a.Hkv, a.Lq, a.L, a.q0, out, a.lse);
   else
     attn_f32_kernel<128><<<static_cast<unsigned>(blocks), kWarps * 32, 0, stream>>>(
-        q, kc, vc, km, vm, a.seed_idx, a.n_seeds, a.B, a.Hq, a.Hkv, a.L, out, a.lse);
+        q, kc, vc, km, vm, a.seed_idx, a.n_seeds, a.B, a.Hq, a.Hkv, a.Lq, a.L, a.q0, out, a.lse);
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
 

@@ -62,7 +62,7 @@ int cover_attn_fwd(const void* q, const void* k_cached, const void* v_cached, co
   if (D != 128) return COVER_ERR_UNSUPPORTED;
   int* st = status_block();
   if (st == nullptr) return COVER_ERR_CUDA;
-  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, L, D, out, lse};
+  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, L, D, out, lse, L, 0};
   return cover::launch_attn_bf16_sm103(a, st, static_cast<cudaStream_t>(stream));
 }
 
@@ -75,7 +75,44 @@ int cover_attn_fwd_f32(const float* q, const float* k_cached, const float* v_cac
   if (D != 64 && D != 128) return COVER_ERR_UNSUPPORTED;
   int* st = status_block();
   if (st == nullptr) return COVER_ERR_CUDA;
-  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, L, D, out, lse};
+  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, L, D, out, lse, L, 0};
+  return cover::launch_attn_f32(a, st, static_cast<cudaStream_t>(stream));
+}
+
+static int check_window(int Lq, int Lk, int q0) {
+  if (Lq < 1 || Lk < 1 || q0 < 0 || static_cast<long long>(q0) + Lq > Lk) return COVER_ERR_INVALID_ARG;
+  return COVER_OK;
+}
+
+int cover_attn_fwd_prefix(const void* q, const void* k_cached, const void* v_cached, const void* k_seedmask,
+                          const void* v_seedmask, const int32_t* seed_idx, int n_seeds, int B, int Hq, int Hkv,
+                          int Lq, int Lk, int q0, int D, void* out, float* lse, void* stream) {
+  int rc = check_window(Lq, Lk, q0);
+  if (rc != COVER_OK) return rc;
+  rc = check_attn_args(q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
+                       16);
+  if (rc != COVER_OK) return rc;
+  if (D != 128) return COVER_ERR_UNSUPPORTED;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
+                    Lq, q0};
+  return cover::launch_attn_bf16_sm103(a, st, static_cast<cudaStream_t>(stream));
+}
+
+int cover_attn_fwd_prefix_f32(const float* q, const float* k_cached, const float* v_cached, const float* k_seedmask,
+                              const float* v_seedmask, const int32_t* seed_idx, int n_seeds, int B, int Hq, int Hkv,
+                              int Lq, int Lk, int q0, int D, float* out, float* lse, void* stream) {
+  int rc = check_window(Lq, Lk, q0);
+  if (rc != COVER_OK) return rc;
+  rc = check_attn_args(q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
+                       4);
+  if (rc != COVER_OK) return rc;
+  if (D != 64 && D != 128) return COVER_ERR_UNSUPPORTED;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
+                    Lq, q0};
   return cover::launch_attn_f32(a, st, static_cast<cudaStream_t>(stream));
 }
 

@@ -16,9 +16,11 @@ struct AttnArgs {
   const void* v_seedmask;
   const int32_t* seed_idx;
   int n_seeds;
-  int B, Hq, Hkv, L, D;
+  int B, Hq, Hkv, L, D;   // L: memory length (keys / values)
   void* out;
   float* lse;
+  int Lq = 0;             // query rows; query row r sits at memory position q0 + r
+  int q0 = 0;
 };
 
 int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream);

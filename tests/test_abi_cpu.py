@@ -142,3 +142,18 @@ def test_seed_kv_no_seeds_is_a_noop(lib):
     # nothing to move: returns before touching the device
     assert lib.cover_seed_kv_override(P, P, None, 0, 2, 2, 16, 128, 2, None, None, None) == 0
     assert lib.cover_seed_kv_gather(P, P, None, 0, 2, 2, 16, 128, 2, None, None, None) == 0
+
+
+@pytest.mark.parametrize("fn", ["cover_attn_fwd_prefix", "cover_attn_fwd_prefix_f32"])
+@pytest.mark.parametrize("kw", [
+    dict(Lq=0), dict(Lk=0), dict(q0=-1), dict(q0=50, Lq=51), dict(n_seeds=101), dict(q=None), dict(Hq=3),
+])
+def test_prefix_invalid_args(lib, fn, kw):
+    a = dict(q=P, kc=P, vc=P, km=P, vm=P, seeds=P, n_seeds=4, B=1, Hq=4, Hkv=2, Lq=50, Lk=100, q0=50, D=128,
+             out=P, lse=None)
+    a.update(kw)
+    assert getattr(lib, fn)(*a.values(), None) == -1
+
+
+def test_prefix_unsupported_head_dim(lib):
+    assert lib.cover_attn_fwd_prefix(P, P, P, P, P, P, 4, 1, 4, 2, 50, 100, 50, 64, P, None, None) == -2
