@@ -106,6 +106,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int hkv = hq / (Hq / Hkv);
   const int row0 = mblk * kRowsPerCta;
   const int nkv = (Lk + kBN - 1) / kBN;
+  // Q tiles holding at least one query row (a short window leaves the second one empty)
+  const int nqt = min(kNQ, (Lq - row0 + kBM - 1) / kBM);
   const int tail_valid = Lk - (nkv - 1) * kBN;   // valid keys in the last KV tile (1..128)
 
   // ---------------- prologue ----------------
@@ -148,8 +150,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_k);
       tma_prefetch_desc(&tm_v);
-      mbar_arrive_expect_tx(&sm.bar_q, kNQ * kTileBytes);
-      for (int t = 0; t < kNQ; ++t)
+      mbar_arrive_expect_tx(&sm.bar_q, nqt * kTileBytes);
+      for (int t = 0; t < nqt; ++t)
         for (int h = 0; h < 2; ++h)
           tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q, 64 * h, row0 + t * kBM, hq, b);
       int last_kj = -1, last_vj = -1;   // last KV tiles whose K / V loads were issued
@@ -199,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // group of products has been queued, so the tensor pipe works while the thread waits.
       for (int j = 0; j <= nkv && ok; ++j) {
         const int st = j & 1, pst = (j - 1) & 1;
-        for (int t = 0; t < kNQ; ++t) {
+        for (int t = 0; t < nqt; ++t) {
           if (j > 0) {
             ok = mbar_wait(&sm.bar_p_full[t], (j - 1) & 1, &sm.abort);
             if (!ok) break;
@@ -211,7 +213,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                       dv0 + pst * kTileDesc + static_cast<uint64_t>((ks * 2048) >> 4), id_pv,
                       (j > 1 || ks > 0) ? 1u : 0u);
             if (j == nkv) umma_commit(&sm.bar_o_full[t]);
-            if (t == kNQ - 1) umma_commit(&sm.bar_v_empty[pst]);
+            if (t == nqt - 1) umma_commit(&sm.bar_v_empty[pst]);
           }
           if (j < nkv) {
             if (t == 0) {
@@ -227,7 +229,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                       ks > 0 ? 1u : 0u);
             }
             umma_commit(&sm.bar_s_full[t]);
-            if (t == kNQ - 1) umma_commit(&sm.bar_k_empty[st]);
+            if (t == nqt - 1) umma_commit(&sm.bar_k_empty[st]);
             if (t == 0) {
               // V(j) feeds the P.V products of the next KV step; it was issued long before
               ok = mbar_wait(&sm.bar_v_full[st], (j >> 1) & 1, &sm.abort);
@@ -246,175 +248,179 @@ __global__ void __launch_bounds__(kThreads, 1)
     setmaxnreg_inc<kSoftmaxRegs>();
     // ---------------- softmax (warps 0-7) ----------------
     const int qt = warp >> 2;
-    const int r = tid & (kBM - 1);
-    const uint32_t trow = tbase + (static_cast<uint32_t>((warp & 3) * 32) << 16);
-    const uint32_t s_addr = trow + col_s(qt);
-    const uint32_t o_addr = trow + col_o(qt);
-    const int grow = row0 + qt * kBM + r;
-    const int my_slot = sm.slot[qt * kBM + r];
-    const bool is_seed = my_slot != kNoSlot && grow < Lq;
-    // the diagonal of this row: KV tile and column of memory position q0 + grow
-    const int diag_j = (q0 + grow) / kBN;
-    const int diag_c = (q0 + grow) % kBN;
-    float m_run = -INFINITY, l_run = 0.0f;
-    bool ok = true;
+    // warps of a Q tile with no query rows (a short window) sit this launch out
+    if (qt < nqt) {
+      const int r = tid & (kBM - 1);
+      const uint32_t trow = tbase + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+      const uint32_t s_addr = trow + col_s(qt);
+      const uint32_t o_addr = trow + col_o(qt);
+      const int grow = row0 + qt * kBM + r;
+      const int my_slot = sm.slot[qt * kBM + r];
+      const bool is_seed = my_slot != kNoSlot && grow < Lq;
+      // the diagonal of this row: KV tile and column of memory position q0 + grow
+      const int diag_j = (q0 + grow) / kBN;
+      const int diag_c = (q0 + grow) % kBN;
+      float m_run = -INFINITY, l_run = 0.0f;
+      bool ok = true;
 
-    // Seed rows: score of the masked-input self pair, s_self = q_i . k_i (log2-scaled),
-    // computed up front so its global loads overlap the first tiles; the value row
-    // is prefetched into L2 for the epilogue.
-    float s_self = 0.0f;
-    const size_t mrow = is_seed ? ((static_cast<size_t>(b) * Hkv + hkv) * n_seeds + my_slot) * kD : 0;
-    if (__any_sync(0xffffffffu, is_seed)) {
-      ok = warp_wait(&sm.bar_q, 0, &sm.abort);
-      if (ok && is_seed) {
-        prefetch_l2(v_seedmask + mrow);
-        prefetch_l2(v_seedmask + mrow + 64);
-        const uint4* kmv = reinterpret_cast<const uint4*>(k_seedmask + mrow);
-        float dot[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      // Seed rows: score of the masked-input self pair, s_self = q_i . k_i (log2-scaled),
+      // computed up front so its global loads overlap the first tiles; the value row
+      // is prefetched into L2 for the epilogue.
+      float s_self = 0.0f;
+      const size_t mrow = is_seed ? ((static_cast<size_t>(b) * Hkv + hkv) * n_seeds + my_slot) * kD : 0;
+      if (__any_sync(0xffffffffu, is_seed)) {
+        ok = warp_wait(&sm.bar_q, 0, &sm.abort);
+        if (ok && is_seed) {
+          prefetch_l2(v_seedmask + mrow);
+          prefetch_l2(v_seedmask + mrow + 64);
+          const uint4* kmv = reinterpret_cast<const uint4*>(k_seedmask + mrow);
+          float dot[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-        for (int ch = 0; ch < 16; ++ch) {
-          const int h = ch >> 3, c8 = ch & 7;
-          const uint4 qv = *reinterpret_cast<const uint4*>(sm.q[qt] + h * kBoxBytes + r * 128 + ((c8 ^ (r & 7)) * 16));
-          const uint4 kv = __ldg(kmv + ch);
-          const __nv_bfloat162* qp = reinterpret_cast<const __nv_bfloat162*>(&qv);
-          const __nv_bfloat162* kp = reinterpret_cast<const __nv_bfloat162*>(&kv);
+          for (int ch = 0; ch < 16; ++ch) {
+            const int h = ch >> 3, c8 = ch & 7;
+            const uint4 qv =
+                *reinterpret_cast<const uint4*>(sm.q[qt] + h * kBoxBytes + r * 128 + ((c8 ^ (r & 7)) * 16));
+            const uint4 kv = __ldg(kmv + ch);
+            const __nv_bfloat162* qp = reinterpret_cast<const __nv_bfloat162*>(&qv);
+            const __nv_bfloat162* kp = reinterpret_cast<const __nv_bfloat162*>(&kv);
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 qf = __bfloat1622float2(qp[e]);
-            const float2 kf = __bfloat1622float2(kp[e]);
-            dot[e] = fmaf(qf.x, kf.x, dot[e]);
-            dot[e] = fmaf(qf.y, kf.y, dot[e]);
+            for (int e = 0; e < 4; ++e) {
+              const float2 qf = __bfloat1622float2(qp[e]);
+              const float2 kf = __bfloat1622float2(kp[e]);
+              dot[e] = fmaf(qf.x, kf.x, dot[e]);
+              dot[e] = fmaf(qf.y, kf.y, dot[e]);
+            }
           }
+          s_self = ((dot[0] + dot[1]) + (dot[2] + dot[3])) * scale_log2;
         }
-        s_self = ((dot[0] + dot[1]) + (dot[2] + dot[3])) * scale_log2;
       }
-    }
 
-    for (int j = 0; j < nkv && ok; ++j) {
-      ok = warp_wait(&sm.bar_s_full[qt], j & 1, &sm.abort);
-      if (!ok) break;
-      tc_fence_after_sync();
-      uint32_t raw[4][32];
+      for (int j = 0; j < nkv && ok; ++j) {
+        ok = warp_wait(&sm.bar_s_full[qt], j & 1, &sm.abort);
+        if (!ok) break;
+        tc_fence_after_sync();
+        uint32_t raw[4][32];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(s_addr + 32 * c, raw[c]);
+        for (int c = 0; c < 4; ++c) tmem_ld32(s_addr + 32 * c, raw[c]);
 #pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld_wait(raw[c]);
-      float* s = reinterpret_cast<float*>(&raw[0][0]);
-      if (j == nkv - 1 && tail_valid < kBN) {
+        for (int c = 0; c < 4; ++c) tmem_ld_wait(raw[c]);
+        float* s = reinterpret_cast<float*>(&raw[0][0]);
+        if (j == nkv - 1 && tail_valid < kBN) {
 #pragma unroll
-        for (int c = 0; c < kBN; ++c)
-          if (c >= tail_valid) s[c] = -INFINITY;
-      }
-      if (__any_sync(0xffffffffu, is_seed && j == diag_j)) {
-        // exclusion of the cached diagonal term of a seed row
-        const bool here = is_seed && j == diag_j;
+          for (int c = 0; c < kBN; ++c)
+            if (c >= tail_valid) s[c] = -INFINITY;
+        }
+        if (__any_sync(0xffffffffu, is_seed && j == diag_j)) {
+          // exclusion of the cached diagonal term of a seed row
+          const bool here = is_seed && j == diag_j;
 #pragma unroll
-        for (int c = 0; c < kBN; ++c)
-          if (here && c == diag_c) s[c] = -INFINITY;
-      }
-      // row maximum: four independent 3-input max chains
-      float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
+          for (int c = 0; c < kBN; ++c)
+            if (here && c == diag_c) s[c] = -INFINITY;
+        }
+        // row maximum: four independent 3-input max chains
+        float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
 #pragma unroll
-      for (int c = 4; c + 8 <= kBN; c += 8) {
-        mx0 = fmax3(mx0, s[c], s[c + 1]);
-        mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
-        mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
-        mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
-      }
-      mx0 = fmax3(mx0, s[kBN - 4], s[kBN - 3]);
-      mx1 = fmax3(mx1, s[kBN - 2], s[kBN - 1]);
-      const float m_tile = fmax3(mx0, mx1, fmaxf(mx2, mx3)) * scale_log2;
-      float alpha = 1.0f;
-      bool rescaled = false;
-      if (m_tile > m_run + kRescaleThreshold) {
-        alpha = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m_tile);
-        m_run = m_tile;
-        rescaled = true;
-      }
-      const float m_use = (m_run == -INFINITY) ? 0.0f : m_run;
-      // p = 2^(s * scale - m) on pairs; four independent partial row sums
-      const uint64_t scale2 = f2_pack(scale_log2, scale_log2);
-      const uint64_t negm2 = f2_pack(-m_use, -m_use);
-      uint64_t acc2[4] = {0, 0, 0, 0};
-      uint32_t packed[64];
+        for (int c = 4; c + 8 <= kBN; c += 8) {
+          mx0 = fmax3(mx0, s[c], s[c + 1]);
+          mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
+          mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
+          mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
+        }
+        mx0 = fmax3(mx0, s[kBN - 4], s[kBN - 3]);
+        mx1 = fmax3(mx1, s[kBN - 2], s[kBN - 1]);
+        const float m_tile = fmax3(mx0, mx1, fmaxf(mx2, mx3)) * scale_log2;
+        float alpha = 1.0f;
+        bool rescaled = false;
+        if (m_tile > m_run + kRescaleThreshold) {
+          alpha = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m_tile);
+          m_run = m_tile;
+          rescaled = true;
+        }
+        const float m_use = (m_run == -INFINITY) ? 0.0f : m_run;
+        // p = 2^(s * scale - m) on pairs; four independent partial row sums
+        const uint64_t scale2 = f2_pack(scale_log2, scale_log2);
+        const uint64_t negm2 = f2_pack(-m_use, -m_use);
+        uint64_t acc2[4] = {0, 0, 0, 0};
+        uint32_t packed[64];
 #pragma unroll
-      for (int c = 0; c < 64; ++c) {
-        float t0, t1;
-        f2_unpack(f2_fma(f2_pack(s[2 * c], s[2 * c + 1]), scale2, negm2), t0, t1);
-        const float p0 = ex2_approx(t0);
-        const float p1 = ex2_approx(t1);
-        packed[c] = pack_bf16x2(p0, p1);
-        acc2[c & 3] = f2_add(acc2[c & 3], f2_pack(p0, p1));
-      }
-      float rs[8];
-      f2_unpack(f2_add(acc2[0], acc2[1]), rs[0], rs[1]);
-      f2_unpack(f2_add(acc2[2], acc2[3]), rs[2], rs[3]);
-      const float rowsum = (rs[0] + rs[1]) + (rs[2] + rs[3]);
-      l_run = l_run * alpha + rowsum;
-      tmem_st32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&packed[0]));
-      tmem_st32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&packed[32]));
-      if (j > 0 && __any_sync(0xffffffffu, rescaled)) {
-        // O holds the products of tiles < j (complete: they were issued before S(j))
+        for (int c = 0; c < 64; ++c) {
+          float t0, t1;
+          f2_unpack(f2_fma(f2_pack(s[2 * c], s[2 * c + 1]), scale2, negm2), t0, t1);
+          const float p0 = ex2_approx(t0);
+          const float p1 = ex2_approx(t1);
+          packed[c] = pack_bf16x2(p0, p1);
+          acc2[c & 3] = f2_add(acc2[c & 3], f2_pack(p0, p1));
+        }
+        float rs[8];
+        f2_unpack(f2_add(acc2[0], acc2[1]), rs[0], rs[1]);
+        f2_unpack(f2_add(acc2[2], acc2[3]), rs[2], rs[3]);
+        const float rowsum = (rs[0] + rs[1]) + (rs[2] + rs[3]);
+        l_run = l_run * alpha + rowsum;
+        tmem_st32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&packed[0]));
+        tmem_st32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&packed[32]));
+        if (j > 0 && __any_sync(0xffffffffu, rescaled)) {
+          // O holds the products of tiles < j (complete: they were issued before S(j))
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          uint32_t o[32];
-          tmem_ld32(o_addr + 32 * c, o);
-          tmem_ld_wait(o);
+          for (int c = 0; c < 4; ++c) {
+            uint32_t o[32];
+            tmem_ld32(o_addr + 32 * c, o);
+            tmem_ld_wait(o);
 #pragma unroll
-          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-          tmem_st32(o_addr + 32 * c, o);
-        }
-      }
-      tmem_st_wait();
-      tc_fence_before_sync();
-      mbar_arrive(&sm.bar_p_full[qt]);
-    }
-    if (ok) ok = warp_wait(&sm.bar_o_full[qt], 0, &sm.abort);
-    if (ok) ok = warp_wait(&sm.bar_q, 0, &sm.abort);
-    if (!ok) {
-      if (!sm.abort) raise_abort(sm, status, 30 + qt);
-    } else {
-      tc_fence_after_sync();
-      uint32_t oraw[4][32];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(o_addr + 32 * c, oraw[c]);
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld_wait(oraw[c]);
-      float* o = reinterpret_cast<float*>(&oraw[0][0]);
-      if (is_seed) {
-        // merge the masked-input self term (k_i, v_i) of this seed row
-        const uint4* vmv = reinterpret_cast<const uint4*>(v_seedmask + mrow);
-        const float m2 = fmaxf(m_run, s_self);
-        const float a = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m2);
-        const float pself = ex2_approx(s_self - m2);
-        l_run = l_run * a + pself;
-#pragma unroll
-        for (int ch = 0; ch < 16; ++ch) {
-          const uint4 vv = __ldg(vmv + ch);
-          const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 vf = __bfloat1622float2(vp[e]);
-            o[ch * 8 + 2 * e] = o[ch * 8 + 2 * e] * a + pself * vf.x;
-            o[ch * 8 + 2 * e + 1] = o[ch * 8 + 2 * e + 1] * a + pself * vf.y;
+            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+            tmem_st32(o_addr + 32 * c, o);
           }
         }
-        m_run = m2;
+        tmem_st_wait();
+        tc_fence_before_sync();
+        mbar_arrive(&sm.bar_p_full[qt]);
       }
-      if (grow < Lq) {
-        const float inv = 1.0f / l_run;
-        uint4* dst = reinterpret_cast<uint4*>(out + ((static_cast<size_t>(b) * Hq + hq) * Lq + grow) * kD);
+      if (ok) ok = warp_wait(&sm.bar_o_full[qt], 0, &sm.abort);
+      if (ok) ok = warp_wait(&sm.bar_q, 0, &sm.abort);
+      if (!ok) {
+        if (!sm.abort) raise_abort(sm, status, 30 + qt);
+      } else {
+        tc_fence_after_sync();
+        uint32_t oraw[4][32];
 #pragma unroll
-        for (int ch = 0; ch < 16; ++ch) {
-          uint4 w;
-          w.x = pack_bf16x2(o[ch * 8 + 0] * inv, o[ch * 8 + 1] * inv);
-          w.y = pack_bf16x2(o[ch * 8 + 2] * inv, o[ch * 8 + 3] * inv);
-          w.z = pack_bf16x2(o[ch * 8 + 4] * inv, o[ch * 8 + 5] * inv);
-          w.w = pack_bf16x2(o[ch * 8 + 6] * inv, o[ch * 8 + 7] * inv);
-          dst[ch] = w;
+        for (int c = 0; c < 4; ++c) tmem_ld32(o_addr + 32 * c, oraw[c]);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) tmem_ld_wait(oraw[c]);
+        float* o = reinterpret_cast<float*>(&oraw[0][0]);
+        if (is_seed) {
+          // merge the masked-input self term (k_i, v_i) of this seed row
+          const uint4* vmv = reinterpret_cast<const uint4*>(v_seedmask + mrow);
+          const float m2 = fmaxf(m_run, s_self);
+          const float a = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m2);
+          const float pself = ex2_approx(s_self - m2);
+          l_run = l_run * a + pself;
+#pragma unroll
+          for (int ch = 0; ch < 16; ++ch) {
+            const uint4 vv = __ldg(vmv + ch);
+            const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 vf = __bfloat1622float2(vp[e]);
+              o[ch * 8 + 2 * e] = o[ch * 8 + 2 * e] * a + pself * vf.x;
+              o[ch * 8 + 2 * e + 1] = o[ch * 8 + 2 * e + 1] * a + pself * vf.y;
+            }
+          }
+          m_run = m2;
         }
-        if (lse != nullptr)
-          lse[(static_cast<size_t>(b) * Hq + hq) * Lq + grow] = (m_run + log2f(l_run)) * 0.6931471805599453f;
+        if (grow < Lq) {
+          const float inv = 1.0f / l_run;
+          uint4* dst = reinterpret_cast<uint4*>(out + ((static_cast<size_t>(b) * Hq + hq) * Lq + grow) * kD);
+#pragma unroll
+          for (int ch = 0; ch < 16; ++ch) {
+            uint4 w;
+            w.x = pack_bf16x2(o[ch * 8 + 0] * inv, o[ch * 8 + 1] * inv);
+            w.y = pack_bf16x2(o[ch * 8 + 2] * inv, o[ch * 8 + 3] * inv);
+            w.z = pack_bf16x2(o[ch * 8 + 4] * inv, o[ch * 8 + 5] * inv);
+            w.w = pack_bf16x2(o[ch * 8 + 6] * inv, o[ch * 8 + 7] * inv);
+            dst[ch] = w;
+          }
+          if (lse != nullptr)
+            lse[(static_cast<size_t>(b) * Hq + hq) * Lq + grow] = (m_run + log2f(l_run)) * 0.6931471805599453f;
+        }
       }
     }
   }
@@ -452,7 +458,8 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
   attn_bf16_kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
       tq, tk, tv, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
-      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, scale_log2, static_cast<__nv_bfloat16*>(a.out), a.lse,
+      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, scale_log2, static_cast<__nv_bfloat16*>(a.out),
+      a.lse,
       status);
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
