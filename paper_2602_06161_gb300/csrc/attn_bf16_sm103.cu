@@ -88,11 +88,15 @@ __device__ __forceinline__ void raise_abort(AttnSmem& sm, int* status, int site)
   sm.abort = 1;
 }
 
+// NQ: Q tiles holding query rows (1 for a window of at most 128 rows, else 2).
+// kWindow: query row r sits at memory position q0 + r of an Lk-long memory;
+// otherwise Lq = Lk and q0 = 0 are compile-time facts.
+template <int NQ, bool kWindow>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ CUtensorMap tm_v, const __nv_bfloat16* __restrict__ k_seedmask,
                      const __nv_bfloat16* __restrict__ v_seedmask, const int32_t* __restrict__ seed_idx, int n_seeds,
-                     int Hq, int Hkv, int Lq, int Lk, int q0, int n_mblk, float scale_log2,
+                     int Hq, int Hkv, int Lq_arg, int Lk, int q0_arg, int n_mblk, float scale_log2,
                      __nv_bfloat16* __restrict__ out,
                      float* __restrict__ lse, int* status) {
   extern __shared__ uint8_t smem_raw[];
@@ -106,8 +110,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int hkv = hq / (Hq / Hkv);
   const int row0 = mblk * kRowsPerCta;
   const int nkv = (Lk + kBN - 1) / kBN;
-  // Q tiles holding at least one query row (a short window leaves the second one empty)
-  const int nqt = min(kNQ, (Lq - row0 + kBM - 1) / kBM);
+  constexpr int nqt = NQ;
+  const int Lq = kWindow ? Lq_arg : Lk;
+  const int q0 = kWindow ? q0_arg : 0;
   const int tail_valid = Lk - (nkv - 1) * kBN;   // valid keys in the last KV tile (1..128)
 
   // ---------------- prologue ----------------
@@ -248,7 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     setmaxnreg_inc<kSoftmaxRegs>();
     // ---------------- softmax (warps 0-7) ----------------
     const int qt = warp >> 2;
-    // warps of a Q tile with no query rows (a short window) sit this launch out
+    // with a single Q tile the second tile's warps sit this launch out
     if (qt < nqt) {
       const int r = tid & (kBM - 1);
       const uint32_t trow = tbase + (static_cast<uint32_t>((warp & 3) * 32) << 16);
@@ -257,9 +262,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int grow = row0 + qt * kBM + r;
       const int my_slot = sm.slot[qt * kBM + r];
       const bool is_seed = my_slot != kNoSlot && grow < Lq;
-      // the diagonal of this row: KV tile and column of memory position q0 + grow
-      const int diag_j = (q0 + grow) / kBN;
-      const int diag_c = (q0 + grow) % kBN;
+      // the diagonal of a square launch is column r of KV tile (row0 + qt * 128) / 128; in a
+      // window a warp's 32 consecutive rows meet their diagonals in at most two KV tiles
+      const int diag_j = kWindow ? (q0 + grow) / kBN : (row0 + qt * kBM) / kBN;
+      const int diag_c = kWindow ? (q0 + grow) % kBN : r;
+      const bool warp_seed = __any_sync(0xffffffffu, is_seed);
+      const int dj_lo = kWindow ? __shfl_sync(0xffffffffu, diag_j, 0) : diag_j;
+      const int dj_hi = kWindow ? __shfl_sync(0xffffffffu, diag_j, 31) : diag_j;
       float m_run = -INFINITY, l_run = 0.0f;
       bool ok = true;
 
@@ -310,7 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < kBN; ++c)
             if (c >= tail_valid) s[c] = -INFINITY;
         }
-        if (__any_sync(0xffffffffu, is_seed && j == diag_j)) {
+        if (warp_seed && (j == dj_lo || j == dj_hi)) {
           // exclusion of the cached diagonal term of a seed row
           const bool here = is_seed && j == diag_j;
 #pragma unroll
@@ -446,17 +455,22 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
   const size_t smem = sizeof(AttnSmem) + 1024;
   static bool attr_set = false;
   if (!attr_set) {
-    if (cudaFuncSetAttribute(attn_bf16_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
-        cudaSuccess)
-      return -3;
-    // the register split inside the kernel assumes exactly kLaunchRegs per thread at launch;
-    // any other count could leave setmaxnreg.inc waiting, so refuse to launch
-    cudaFuncAttributes fa;
-    if (cudaFuncGetAttributes(&fa, attn_bf16_kernel) != cudaSuccess || fa.numRegs != kLaunchRegs) return -2;
+    for (auto fn : {attn_bf16_kernel<2, false>, attn_bf16_kernel<1, true>, attn_bf16_kernel<2, true>}) {
+      if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
+        return -3;
+      // the register split inside the kernel assumes exactly kLaunchRegs per thread at launch;
+      // any other count could leave setmaxnreg.inc waiting, so refuse to launch
+      cudaFuncAttributes fa;
+      if (cudaFuncGetAttributes(&fa, fn) != cudaSuccess || fa.numRegs != kLaunchRegs) return -2;
+    }
     attr_set = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
-  attn_bf16_kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
+  const bool window = a.Lq != a.L || a.q0 != 0;
+  auto kernel = !window       ? attn_bf16_kernel<2, false>
+                : a.Lq <= kBM ? attn_bf16_kernel<1, true>
+                              : attn_bf16_kernel<2, true>;
+  kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
       tq, tk, tv, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
       a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, scale_log2, static_cast<__nv_bfloat16*>(a.out),
       a.lse,
