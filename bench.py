@@ -16,6 +16,8 @@ Printed JSON line (rank 0):
   decide       scoring fused with one step's decisions (drafting, revision,
                adaptive seed selection) against scoring + top-k alone
   seed_kv      per-layer seed K/V cache gather and override swap
+  prefix_window  the attention of the last block's query rows over the full
+               memory (prefix-cache decoding)
   cpu_baseline the fp64 oracle on a bounded sample of the same workload
 
 ``--impl reference`` times the fp64 oracle (the only reference there is: the
@@ -349,6 +351,7 @@ def run_ours(args):
     if not args.no_secondary:
         per = {WORKLOAD: seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops)}
         kv_all = {WORKLOAD: kv_timing(api, torch, kc, vc, seeds)}
+        prefix_all = {WORKLOAD: prefix_timing(api, torch, q, kc, vc, km, vm, seeds, 64, peak)}
         del q, kc, vc, km, vm, logits
         torch.cuda.empty_cache()
         scoring_all = {WORKLOAD: scoring["gbs"]}
@@ -362,6 +365,8 @@ def run_ours(args):
             olse = torch.empty((ow.B, ow.Hq, ow.L), dtype=torch.float32, device="cuda")
             per[name] = seed_overhead(api, torch, oq, okc, ovc, okm, ovm, oseeds, oout, olse, ow.attn_flops)
             kv_all[name] = kv_timing(api, torch, okc, ovc, oseeds)
+            if name == "dream_gqa_l1024":
+                prefix_all[name] = prefix_timing(api, torch, oq, okc, ovc, okm, ovm, oseeds, 32, peak)
             del oq, okc, ovc, okm, ovm, oseeds, oout, olse
             osi = ow.score_inputs()
             if osi is not None:
@@ -374,6 +379,7 @@ def run_ours(args):
                                   "peak_source": roofline["peak_source"]}
         result["scoring_gbs"] = scoring_all
         result["seed_kv"] = kv_all
+        result["prefix_window"] = prefix_all
         result["decide"] = {name: decide_timing(api, torch, W.WORKLOADS[name])
                             for name in (WORKLOAD, "dream_gqa_l1024")}
         status = api.cover_device_status()
@@ -467,6 +473,31 @@ def decide_timing(api, torch, wl, iters=20):
             "gbs": round(nbytes / (t_dec * 1e-3) / 1e9, 1),
             "drafted_per_seq": round(float(stats[:, 0].mean()), 2),
             "seeds_per_seq": round(float(out["n_seeds"].float().mean().item()), 2)}
+
+
+def prefix_timing(api, torch, q, kc, vc, km, vm, seeds, Lq, peak, iters=20):
+    """Prefix-cache window (Section 6.6): the last Lq query rows (the active block) over the full memory."""
+    B, Hq, L, D = q.shape
+    q0 = L - Lq
+    qw = q[:, :, q0:].contiguous()
+    out = torch.empty_like(qw)
+    lse = torch.empty((B, Hq, Lq), dtype=torch.float32, device=q.device)
+    stream = torch.cuda.current_stream()
+    for _ in range(3):
+        api.cover_attn_fwd_prefix(qw, kc, vc, km, vm, seeds, q0=q0, out=out, lse=lse)
+    ts = []
+    for _ in range(iters):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        busy_ahead(torch)
+        a.record(stream)
+        api.cover_attn_fwd_prefix(qw, kc, vc, km, vm, seeds, q0=q0, out=out, lse=lse)
+        b.record(stream)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    t = statistics.median(ts)
+    flops = 4.0 * B * Hq * Lq * L * D
+    return {"Lq": Lq, "Lk": L, "q0": q0, "ms": round(t, 4), "tflops": round(flops / (t * 1e-3) / 1e12, 2),
+            "frac_of_peak": round(flops / (t * 1e-3) / 1e12 / peak, 4)}
 
 
 def kv_timing(api, torch, k, v, seeds, iters=20):
