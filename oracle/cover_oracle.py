@@ -23,6 +23,8 @@ Everything here is written from the paper's definitions:
   Keep / Replace / ReMask revision of the previous seeds, the state update;
   §5.3: the seed score on the updated state, the adaptive revision rate
   |S_t| = ceil(sqrt(n_t pi_t)) and the exclusions from seed selection.
+* §5.3 (d_in, d_out): attention mass from masked queries into a position and
+  from a position into the drafted ones, over the head-averaged weights.
 * §5.1 (seed K/V cache): the states of the new seeds cached at selection and
   written over the seed columns of the next step's memory, the masked-input
   states moving into the diagonal side buffer.
@@ -211,6 +213,47 @@ def override_attention_window(q, kc, vc, km, vm, seed_idx, q0: int):
                 K, V = view_for_row(kc[b, hkv], vc[b, hkv], i, pair)
                 out[b, hq, r], lse[b, hq, r], _ = attention_row(q[b, hq, r], K, V)
     return out, lse
+
+
+def attention_mass(q, kc, km, seed_idx, masked, drafted, pos0: int):
+    """d_in and d_out of §5.3 from the head-averaged attention of the current pass.
+
+    q [B,Hq,L,D] and kc [B,Hkv,L,D] (= K') cover every memory position; km
+    [B,Hkv,S,D] holds the masked-input keys of the seeds (seed_idx [B,S]).
+    The weight row of a query is its softmax over its own key set (§5.1: K',
+    with the diagonal restored to k_i for a seed), i.e. the corrected weights
+    of App. B.3. A = mean over the Hq heads of those weight matrices.
+    masked / drafted [B, n] flag the response positions pos0 .. pos0+n-1 that
+    are in M_t (masked after the update) and D_t (drafted this step). Returns
+    d_in, d_out [B, n]: d_in[j] = sum over masked q of A[q -> j], d_out[j] =
+    sum over drafted i of A[j -> i], for the response positions j.
+    """
+    B, Hq, L, D = q.shape
+    Hkv = kc.shape[1]
+    G = Hq // Hkv
+    n = masked.shape[1]
+    S = 0 if seed_idx is None else seed_idx.shape[1]
+    slot = route_seeds(seed_idx, L)[0] if S else np.full((B, L), -1, np.int32)
+    d_in = np.zeros((B, n))
+    d_out = np.zeros((B, n))
+    for b in range(B):
+        A = np.zeros((n, L))                       # head-averaged weight rows of the response queries
+        for hq in range(Hq):
+            hkv = hq // G
+            for r in range(n):
+                i = pos0 + r
+                s = int(slot[b, i])
+                K = kc[b, hkv]
+                if s >= 0:
+                    K = K.copy()
+                    K[i] = km[b, hkv, s]
+                z = K @ q[b, hq, i] / math.sqrt(D)
+                w = np.exp(z - z.max())
+                A[r] += w / w.sum() / Hq
+        cols = A[:, pos0:pos0 + n]                 # attention from response queries to response keys
+        d_in[b] = cols[np.asarray(masked[b], bool)].sum(axis=0)
+        d_out[b] = cols[:, np.asarray(drafted[b], bool)].sum(axis=1)
+    return d_in, d_out
 
 
 def override_attention_closed_form(q, kc, vc, km, vm, seed_idx):

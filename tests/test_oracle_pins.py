@@ -449,3 +449,51 @@ def test_window_with_seeds_outside_is_plain_attention():
     out, lse = oracle.override_attention_window(q[:, :, 5:15], kc, vc, km, vm, seeds, 5)
     ref, ref_lse = sdpa_reference(q[:, :, 5:15], kc, vc)
     assert np.max(np.abs(out - ref)) < 1e-12 and np.max(np.abs(lse - ref_lse)) < 1e-12
+
+
+# ----------------------------------------------------------------------------
+# d_in / d_out (Section 5.3) from the head-averaged attention weights
+# ----------------------------------------------------------------------------
+
+def test_mass_sums_to_the_counts():
+    # each weight row sums to 1: over the whole memory (pos0 = 0, every position a response
+    # position) the total incoming mass is |M_t|, and a position whose every key is drafted
+    # sends mass 1
+    rng = np.random.default_rng(50)
+    q, kc, vc, km, vm, seeds = rand_case(2, 4, 2, 12, 8, 3, rng=rng)
+    masked = rng.random((2, 12)) < 0.4
+    d_in, d_out = oracle.attention_mass(q, kc, km, seeds, masked, np.ones((2, 12), bool), 0)
+    assert np.allclose(d_in.sum(axis=1), masked.sum(axis=1), atol=1e-12)
+    assert np.allclose(d_out, 1.0, atol=1e-12)
+    d_in, d_out = oracle.attention_mass(q, kc, km, seeds, np.zeros((2, 12), bool), np.zeros((2, 12), bool), 0)
+    assert not d_in.any() and not d_out.any()
+
+
+def test_mass_uniform_queries():
+    # q = 0: every weight is 1/L (seed rows too), so d_in = |M|/L and d_out = |D|/L
+    rng = np.random.default_rng(51)
+    _, kc, vc, km, vm, seeds = rand_case(1, 2, 1, 10, 4, 2, rng=rng)
+    q = np.zeros((1, 2, 10, 4))
+    masked = np.zeros((1, 6), bool)
+    masked[0, [1, 4]] = True
+    drafted = np.zeros((1, 6), bool)
+    drafted[0, [0, 2, 5]] = True
+    d_in, d_out = oracle.attention_mass(q, kc, km, seeds, masked, drafted, 3)
+    assert np.allclose(d_in, 2 / 10, atol=1e-15) and np.allclose(d_out, 3 / 10, atol=1e-15)
+
+
+def test_mass_matches_the_corrected_weights():
+    # the weight rows are App. B.3's corrected weights (pinned above): sum them directly
+    rng = np.random.default_rng(52)
+    q, kc, vc, km, vm, seeds = rand_case(1, 2, 2, 9, 4, 3, rng=rng)
+    pos0, n = 2, 6
+    masked = rng.random((1, n)) < 0.5
+    drafted = rng.random((1, n)) < 0.5
+    d_in, d_out = oracle.attention_mass(q, kc, km, seeds, masked, drafted, pos0)
+    A = np.zeros((n, 9))
+    for hq in range(2):
+        for r in range(n):
+            A[r] += oracle.corrected_weights_row(q, kc, vc, km, vm, seeds, 0, hq, pos0 + r) / 2
+    for j in range(n):
+        assert abs(d_in[0, j] - sum(A[r, pos0 + j] for r in range(n) if masked[0, r])) < 1e-12
+        assert abs(d_out[0, j] - sum(A[j, pos0 + i] for i in range(n) if drafted[0, i])) < 1e-12
