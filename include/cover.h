@@ -271,20 +271,79 @@ int cover_seed_kv_override(void* k, void* v, const int32_t* seed_idx, int n_seed
  * workspace: cover_decide_workspace_bytes(N, n_seq) bytes of device memory,
  *          16-byte aligned, zero-filled before its first use; it is left ready
  *          for the next call on the same stream.
+ * phase COVER_DECIDE_ALL runs steps 1-5 with the given d_in / d_out.
+ * phase COVER_DECIDE_UPDATE runs steps 1-2 only: it writes maxprob, entropy,
+ *   argmax, the updated tok / remask_cnt, flag bit COVER_FLAG_DRAFTED on the
+ *   rows drafted in this step (bit COVER_FLAG_SEED still marks the previous
+ *   seeds), stats[.., 0..3], and the uncertainty of every row's updated token
+ *   into the workspace; score, seed_idx and n_seeds are not written (they may
+ *   be NULL). Then cover_attn_mass_fwd produces d_in / d_out from the updated
+ *   state, and cover_seed_select_fwd runs steps 3-5 on the same workspace. This
+ *   is the order of Section 5.3, where d_in sums over the masked positions after
+ *   the update and d_out over the positions drafted in this step.
  * Errors: COVER_ERR_INVALID_ARG for a NULL required pointer, N, V or n_seq < 1,
  * N % n_seq != 0, N / n_seq > 4096, draft_budget, remask_budget or max_seeds
- * < 0, or a misaligned pointer. COVER_ERR_CUDA for a launch failure.
+ * < 0, an unknown phase, or a misaligned pointer. COVER_ERR_CUDA for a launch
+ * failure.
  */
 #define COVER_FLAG_SEED 1
+#define COVER_FLAG_DRAFTED 2
+#define COVER_DECIDE_ALL 0
+#define COVER_DECIDE_UPDATE 1
 size_t cover_decide_workspace_bytes(int N, int n_seq);
 int cover_score_decide_fwd(const void* logits, int N, int V, int n_seq,
                            const float* d_in, const float* d_out, const uint8_t* draft_ok,
                            float tau_draft, int draft_budget, int remask_budget, int mask_id,
-                           int min_one, int pos0, int max_seeds,
+                           int min_one, int pos0, int max_seeds, int phase,
                            int32_t* tok, uint8_t* flags, uint8_t* remask_cnt,
                            float* maxprob, float* entropy, int32_t* argmax, float* score,
                            int32_t* seed_idx, int32_t* n_seeds, int32_t* stats,
                            void* workspace, void* stream);
+
+/*
+ * d_in and d_out of the seed score (Section 5.3) from the attention of the
+ * current pass, averaged over the Hq heads: for the response positions
+ * pos0 .. pos0 + per - 1 of every batch row (state row b * per + i is
+ * position pos0 + i),
+ *   d_in(j)  = sum over masked positions q (tok == mask_id) of A[q -> j],
+ *   d_out(j) = sum over positions i with flag bit COVER_FLAG_DRAFTED of A[j -> i],
+ * where A_h[q -> j] = exp(q_q . k'_j / sqrt(D) - lse_h(q)) and a seed query's
+ * diagonal uses its masked-input key (the leave-one-out view; lse is the one
+ * cover_attn_fwd wrote, that of the corrected distribution). Only response
+ * queries and response keys contribute. Tensor-core recomputation of the
+ * per x per block of every head; partial sums per head are added in a fixed
+ * order, so the result is deterministic.
+ * q [B, Hq, L, 128], k_cached [B, Hkv, L, 128], k_seedmask [B, Hkv, n_seeds,
+ * 128] bf16; seed_idx int32 [B, n_seeds]; lse float [B, Hq, L]; tok int32,
+ * flags uint8 [B * per] (cover_score_decide_fwd's state after the update
+ * phase); d_in, d_out float [B * per] (out). workspace:
+ * cover_attn_mass_workspace_bytes(B, Hq, per) bytes, 16-byte aligned, no
+ * initialisation needed. All device pointers, owned by the caller.
+ * Errors: COVER_ERR_INVALID_ARG for a NULL required pointer, B, Hq, Hkv, L,
+ * per < 1, Hq % Hkv != 0, pos0 < 0 or pos0 + per > L, n_seeds < 0 or > L, or a
+ * misaligned pointer; COVER_ERR_UNSUPPORTED for D != 128; COVER_ERR_CUDA for a
+ * launch failure; COVER_ERR_DEVICE_TIMEOUT via cover_device_status.
+ */
+size_t cover_attn_mass_workspace_bytes(int B, int Hq, int per);
+int cover_attn_mass_fwd(const void* q, const void* k_cached, const void* k_seedmask,
+                        const int32_t* seed_idx, int n_seeds, const float* lse,
+                        int B, int Hq, int Hkv, int L, int D,
+                        const int32_t* tok, const uint8_t* flags, int mask_id, int pos0, int per,
+                        void* workspace, float* d_in, float* d_out, void* stream);
+
+/*
+ * Steps 3-5 of cover_score_decide_fwd (seed score, adaptive revision rate,
+ * selection) after a COVER_DECIDE_UPDATE call on the same workspace and state:
+ * score = u * (1 + d_in) / (1 + d_out) with u of the updated token; clears flag
+ * bits COVER_FLAG_SEED and COVER_FLAG_DRAFTED, then sets COVER_FLAG_SEED on the
+ * new seeds; writes score [N], seed_idx [n_seq, max_seeds], n_seeds [n_seq] and
+ * stats[.., 4..5]. Arguments and errors as cover_score_decide_fwd.
+ */
+int cover_seed_select_fwd(int N, int n_seq, const float* d_in, const float* d_out,
+                          int remask_budget, int mask_id, int pos0, int max_seeds,
+                          int32_t* tok, uint8_t* flags, uint8_t* remask_cnt, float* score,
+                          int32_t* seed_idx, int32_t* n_seeds, int32_t* stats,
+                          void* workspace, void* stream);
 
 /*
  * Synchronises `stream`, then returns and clears the current device's status

@@ -29,8 +29,11 @@ _SIGNATURES = {
     "cover_seed_kv_gather": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
     "cover_seed_kv_override": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
     "cover_decide_workspace_bytes": (ctypes.c_size_t, [_I, _I]),
-    "cover_score_decide_fwd": (_I, [_P, _I, _I, _I, _P, _P, _P, ctypes.c_float, _I, _I, _I, _I, _I, _I,
+    "cover_score_decide_fwd": (_I, [_P, _I, _I, _I, _P, _P, _P, ctypes.c_float, _I, _I, _I, _I, _I, _I, _I,
                                     _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P]),
+    "cover_seed_select_fwd": (_I, [_I, _I, _P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P]),
+    "cover_attn_mass_workspace_bytes": (ctypes.c_size_t, [_I, _I, _I]),
+    "cover_attn_mass_fwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _P, _P, _I, _I, _I, _P, _P, _P, _P]),
     "cover_device_status": (_I, [_P]),
     "cover_status_str": (ctypes.c_char_p, [_I]),
     "cover_debug_umma_tile": (_I, [_P, _P, _P, _P, _P, _P, _P]),

@@ -284,16 +284,23 @@ def decide_workspace(N: int, n_seq: int, device=None) -> torch.Tensor:
     return torch.zeros((max(nbytes, 16) + 15) // 16, 4, dtype=torch.int32, device=device or "cuda")
 
 
+COVER_DECIDE_ALL = 0
+COVER_DECIDE_UPDATE = 1
+
+
 def cover_score_decide_fwd(logits, n_seq: int, tok, flags, remask_cnt, *, tau_draft: float, draft_budget: int,
                            remask_budget: int, mask_id: int, min_one: bool = True, pos0: int = 0,
-                           max_seeds: int = 0, d_in=None, d_out=None, draft_ok=None, workspace=None, out=None,
-                           stream=None):
+                           max_seeds: int = 0, phase: int = COVER_DECIDE_ALL, d_in=None, d_out=None, draft_ok=None,
+                           workspace=None, out=None, stream=None):
     """Scoring fused with one decoding step's decisions (drafting, revision, seed selection).
 
     tok (int32 [N]), flags and remask_cnt (uint8 [N]) are updated in place.
     Returns a dict of CUDA tensors: maxprob, entropy, argmax, score [N];
     seed_idx [n_seq, max_seeds] (positions, -1 padded), n_seeds [n_seq] and
     stats [n_seq, 6] (drafted, kept, replaced, remasked, n_t, n_above).
+    With phase=COVER_DECIDE_UPDATE only drafting, revision and the state update
+    run (score, seed_idx and n_seeds are left as they are); cover_attn_mass_fwd
+    and cover_seed_select_fwd on the same workspace complete the step.
     """
     _need(logits, "logits", torch.bfloat16, 2)
     N, V = logits.shape
@@ -319,12 +326,82 @@ def cover_score_decide_fwd(logits, n_seq: int, tok, flags, remask_cnt, *, tau_dr
         workspace = decide_workspace(N, n_seq, dev)
     code = _lib.load().cover_score_decide_fwd(
         _ptr(logits), N, V, n_seq, _ptr(d_in), _ptr(d_out), _ptr(draft_ok), float(tau_draft), int(draft_budget),
-        int(remask_budget), int(mask_id), 1 if min_one else 0, int(pos0), int(max_seeds),
+        int(remask_budget), int(mask_id), 1 if min_one else 0, int(pos0), int(max_seeds), int(phase),
         _ptr(tok), _ptr(flags), _ptr(remask_cnt), _ptr(out["maxprob"]), _ptr(out["entropy"]), _ptr(out["argmax"]),
         _ptr(out["score"]), _ptr(out["seed_idx"]) if max_seeds > 0 else None, _ptr(out["n_seeds"]),
         _ptr(out["stats"]), _ptr(workspace), _stream(stream))
     _lib.check("cover_score_decide_fwd", code)
     return out
+
+
+def cover_seed_select_fwd(n_seq: int, tok, flags, remask_cnt, workspace, *, remask_budget: int, mask_id: int,
+                          pos0: int = 0, max_seeds: int = 0, d_in=None, d_out=None, out=None, stream=None):
+    """Seed score, adaptive revision rate and selection after a COVER_DECIDE_UPDATE call.
+
+    `workspace` and the state tensors must be those of that call. Returns a
+    dict of CUDA tensors: score [N], seed_idx [n_seq, max_seeds], n_seeds
+    [n_seq], stats [n_seq, 6] (columns 4-5 written here).
+    """
+    _need(tok, "tok", torch.int32, 1)
+    _need(flags, "flags", torch.uint8, 1)
+    _need(remask_cnt, "remask_cnt", torch.uint8, 1)
+    N = tok.shape[0]
+    dev = tok.device
+    for name, t in (("d_in", d_in), ("d_out", d_out)):
+        if t is not None:
+            _need(t, name, torch.float32, 1)
+    if out is None:
+        out = dict(score=torch.empty(N, dtype=torch.float32, device=dev),
+                   seed_idx=torch.empty((n_seq, max(max_seeds, 0)), dtype=torch.int32, device=dev),
+                   n_seeds=torch.empty(n_seq, dtype=torch.int32, device=dev),
+                   stats=torch.zeros((n_seq, 6), dtype=torch.int32, device=dev))
+    code = _lib.load().cover_seed_select_fwd(
+        N, n_seq, _ptr(d_in), _ptr(d_out), int(remask_budget), int(mask_id), int(pos0), int(max_seeds),
+        _ptr(tok), _ptr(flags), _ptr(remask_cnt), _ptr(out["score"]),
+        _ptr(out["seed_idx"]) if max_seeds > 0 else None, _ptr(out["n_seeds"]), _ptr(out["stats"]),
+        _ptr(workspace), _stream(stream))
+    _lib.check("cover_seed_select_fwd", code)
+    return out
+
+
+def cover_attn_mass_workspace_bytes(B: int, Hq: int, per: int) -> int:
+    return int(_lib.load().cover_attn_mass_workspace_bytes(int(B), int(Hq), int(per)))
+
+
+def cover_attn_mass_fwd(q, k_cached, lse, tok, flags, *, mask_id: int, pos0: int, per: int, k_seedmask=None,
+                        seed_idx=None, workspace=None, d_in=None, d_out=None, stream=None):
+    """d_in / d_out (Section 5.3) of the response rows from the attention pass's q, K', lse.
+
+    q [B, Hq, L, 128], k_cached [B, Hkv, L, 128] bf16, lse [B, Hq, L] f32 (as
+    cover_attn_fwd wrote it), tok int32 / flags uint8 [B * per] (the state
+    after a COVER_DECIDE_UPDATE call). Returns (d_in, d_out), float32 [B * per].
+    """
+    _need(q, "q", torch.bfloat16, 4)
+    _need(k_cached, "k_cached", torch.bfloat16, 4)
+    _need(lse, "lse", torch.float32, 3)
+    _need(tok, "tok", torch.int32, 1)
+    _need(flags, "flags", torch.uint8, 1)
+    B, Hq, L, D = q.shape
+    Hkv = k_cached.shape[1]
+    n_seeds = 0 if seed_idx is None else int(seed_idx.shape[1])
+    if n_seeds > 0:
+        _need(seed_idx, "seed_idx", torch.int32, 2)
+        _need(k_seedmask, "k_seedmask", torch.bfloat16, 4)
+    if tok.shape[0] != B * per or flags.shape[0] != B * per:
+        raise ValueError("tok / flags must have B * per entries")
+    if workspace is None:
+        nbytes = cover_attn_mass_workspace_bytes(B, Hq, per)
+        workspace = torch.empty((nbytes + 15) // 16, 4, dtype=torch.int32, device=q.device)
+    if d_in is None:
+        d_in = torch.empty(B * per, dtype=torch.float32, device=q.device)
+    if d_out is None:
+        d_out = torch.empty(B * per, dtype=torch.float32, device=q.device)
+    code = _lib.load().cover_attn_mass_fwd(
+        _ptr(q), _ptr(k_cached), _ptr(k_seedmask) if n_seeds else None, _ptr(seed_idx) if n_seeds else None,
+        n_seeds, _ptr(lse), B, Hq, Hkv, L, D, _ptr(tok), _ptr(flags), int(mask_id), int(pos0), int(per),
+        _ptr(workspace), _ptr(d_in), _ptr(d_out), _stream(stream))
+    _lib.check("cover_attn_mass_fwd", code)
+    return d_in, d_out
 
 
 def cover_device_status(stream=None) -> int:

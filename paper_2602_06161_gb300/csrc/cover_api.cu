@@ -208,15 +208,19 @@ size_t cover_decide_workspace_bytes(int N, int n_seq) {
 
 int cover_score_decide_fwd(const void* logits, int N, int V, int n_seq, const float* d_in, const float* d_out,
                            const uint8_t* draft_ok, float tau_draft, int draft_budget, int remask_budget,
-                           int mask_id, int min_one, int pos0, int max_seeds, int32_t* tok, uint8_t* flags,
-                           uint8_t* remask_cnt, float* maxprob, float* entropy, int32_t* argmax, float* score,
-                           int32_t* seed_idx, int32_t* n_seeds, int32_t* stats, void* workspace, void* stream) {
+                           int mask_id, int min_one, int pos0, int max_seeds, int phase, int32_t* tok,
+                           uint8_t* flags, uint8_t* remask_cnt, float* maxprob, float* entropy, int32_t* argmax,
+                           float* score, int32_t* seed_idx, int32_t* n_seeds, int32_t* stats, void* workspace,
+                           void* stream) {
+  if (phase != COVER_DECIDE_ALL && phase != COVER_DECIDE_UPDATE) return COVER_ERR_INVALID_ARG;
+  const bool select = phase == COVER_DECIDE_ALL;
   if (logits == nullptr || tok == nullptr || flags == nullptr || remask_cnt == nullptr || maxprob == nullptr ||
-      entropy == nullptr || argmax == nullptr || score == nullptr || n_seeds == nullptr || workspace == nullptr)
+      entropy == nullptr || argmax == nullptr || workspace == nullptr)
     return COVER_ERR_INVALID_ARG;
+  if (select && (score == nullptr || n_seeds == nullptr)) return COVER_ERR_INVALID_ARG;
   if (N < 1 || V < 1 || n_seq < 1 || N % n_seq != 0 || N / n_seq > 4096) return COVER_ERR_INVALID_ARG;
   if (draft_budget < 0 || remask_budget < 0 || max_seeds < 0) return COVER_ERR_INVALID_ARG;
-  if (max_seeds > 0 && seed_idx == nullptr) return COVER_ERR_INVALID_ARG;
+  if (select && max_seeds > 0 && seed_idx == nullptr) return COVER_ERR_INVALID_ARG;
   if (!aligned(logits, 16) || !aligned(workspace, 16) || !aligned(tok, 4) || !aligned(maxprob, 4) ||
       !aligned(entropy, 4) || !aligned(argmax, 4) || !aligned(score, 4) || !aligned(n_seeds, 4))
     return COVER_ERR_INVALID_ARG;
@@ -232,8 +236,60 @@ int cover_score_decide_fwd(const void* logits, int N, int V, int n_seq, const fl
   cover::ScoreArgs a{logits, N, V, n_seq, nullptr, d_in, d_out, nullptr, 0, maxprob, entropy, argmax, score,
                      nullptr, nullptr, reinterpret_cast<uint32_t*>(ws)};
   cover::DecideArgs d{draft_ok, tau_draft, draft_budget, remask_budget, mask_id, min_one != 0 ? 1 : 0, pos0,
-                      max_seeds, tok, flags, remask_cnt, seed_idx, n_seeds, stats, ws_u, ws_lnz};
+                      max_seeds, tok, flags, remask_cnt, seed_idx, n_seeds, stats, ws_u, ws_lnz, phase};
   return cover::launch_score_decide(a, d, st, static_cast<cudaStream_t>(stream));
+}
+
+int cover_seed_select_fwd(int N, int n_seq, const float* d_in, const float* d_out, int remask_budget, int mask_id,
+                          int pos0, int max_seeds, int32_t* tok, uint8_t* flags, uint8_t* remask_cnt, float* score,
+                          int32_t* seed_idx, int32_t* n_seeds, int32_t* stats, void* workspace, void* stream) {
+  if (tok == nullptr || flags == nullptr || remask_cnt == nullptr || score == nullptr || n_seeds == nullptr ||
+      workspace == nullptr)
+    return COVER_ERR_INVALID_ARG;
+  if (N < 1 || n_seq < 1 || N % n_seq != 0 || N / n_seq > 4096) return COVER_ERR_INVALID_ARG;
+  if (remask_budget < 0 || max_seeds < 0) return COVER_ERR_INVALID_ARG;
+  if (max_seeds > 0 && seed_idx == nullptr) return COVER_ERR_INVALID_ARG;
+  if (!aligned(workspace, 16) || !aligned(tok, 4) || !aligned(score, 4) || !aligned(n_seeds, 4) ||
+      (seed_idx != nullptr && !aligned(seed_idx, 4)) || (stats != nullptr && !aligned(stats, 4)) ||
+      (d_in != nullptr && !aligned(d_in, 4)) || (d_out != nullptr && !aligned(d_out, 4)))
+    return COVER_ERR_INVALID_ARG;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  const size_t counters_bytes = (sizeof(uint32_t) * static_cast<size_t>(n_seq) + 15) & ~static_cast<size_t>(15);
+  float* ws_u = reinterpret_cast<float*>(ws + counters_bytes);
+  cover::DecideArgs d{nullptr, 0.0f, 0, remask_budget, mask_id, 0, pos0, max_seeds, tok, flags, remask_cnt,
+                      seed_idx, n_seeds, stats, ws_u, ws_u + N, COVER_DECIDE_ALL};
+  return cover::launch_seed_select(N, n_seq, d, d_in, d_out, score, static_cast<cudaStream_t>(stream)) == 0
+             ? COVER_OK
+             : COVER_ERR_CUDA;
+}
+
+size_t cover_attn_mass_workspace_bytes(int B, int Hq, int per) {
+  if (B < 1 || Hq < 1 || per < 1) return 0;
+  return cover::mass_workspace_bytes(B, Hq, per);
+}
+
+int cover_attn_mass_fwd(const void* q, const void* k_cached, const void* k_seedmask, const int32_t* seed_idx,
+                        int n_seeds, const float* lse, int B, int Hq, int Hkv, int L, int D, const int32_t* tok,
+                        const uint8_t* flags, int mask_id, int pos0, int per, void* workspace, float* d_in,
+                        float* d_out, void* stream) {
+  if (q == nullptr || k_cached == nullptr || lse == nullptr || tok == nullptr || flags == nullptr ||
+      workspace == nullptr || d_in == nullptr || d_out == nullptr)
+    return COVER_ERR_INVALID_ARG;
+  if (B < 1 || Hq < 1 || Hkv < 1 || L < 1 || D < 1 || per < 1 || Hq % Hkv != 0) return COVER_ERR_INVALID_ARG;
+  if (pos0 < 0 || static_cast<long long>(pos0) + per > L) return COVER_ERR_INVALID_ARG;
+  if (n_seeds < 0 || n_seeds > L || (n_seeds > 0 && (seed_idx == nullptr || k_seedmask == nullptr)))
+    return COVER_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(k_cached, 16) || !aligned(workspace, 16) || !aligned(lse, 4) ||
+      !aligned(tok, 4) || !aligned(d_in, 4) || !aligned(d_out, 4))
+    return COVER_ERR_INVALID_ARG;
+  if (n_seeds > 0 && (!aligned(k_seedmask, 16) || !aligned(seed_idx, 4))) return COVER_ERR_INVALID_ARG;
+  if (D != 128) return COVER_ERR_UNSUPPORTED;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  cover::MassArgs a{q, k_cached, k_seedmask, seed_idx, n_seeds, lse, B, Hq, Hkv, L, pos0, per, tok, flags,
+                    mask_id, workspace, d_in, d_out};
+  const int rc = cover::launch_attn_mass(a, st, static_cast<cudaStream_t>(stream));
+  return rc == -2 ? COVER_ERR_UNSUPPORTED : rc == 0 ? COVER_OK : COVER_ERR_CUDA;
 }
 
 int cover_device_status(void* stream) {

@@ -66,16 +66,40 @@ struct DecideArgs {
   int32_t* seed_idx;         // [n_seq, max_seeds] positions, -1 padded
   int32_t* n_seeds;          // [n_seq]
   int32_t* stats;            // [n_seq, 6] or null
-  float* ws_u;               // [N] workspace: u of the current token
+  float* ws_u;               // [N] workspace: u of the current token, then of the updated one
   float* ws_lnz;             // [N] workspace: ln Z (= u of the greedy token)
+  int phase = 0;             // 0: update and select; 1: update only (flag bit 1 marks drafted rows)
 };
 constexpr int kDecideStats = 6;   // drafted, kept, replaced, remasked, n_t, n_above
 int launch_score_decide(const ScoreArgs& a, const DecideArgs& d, int* status, cudaStream_t stream);
+// Section 5.3 selection alone, from the state and workspace an update phase left.
+int launch_seed_select(int N, int n_seq, const DecideArgs& d, const float* d_in, const float* d_out, float* score,
+                       cudaStream_t stream);
 
 // Same as launch_score, with the counters in a fixed device array of the
 // library (a.counters is ignored). Returns -1 if a.n_seq > kNoAllocMaxSegments.
 constexpr int kNoAllocMaxSegments = 4096;
 int launch_score_noalloc(ScoreArgs a, int* status, cudaStream_t stream);
+
+// d_in / d_out of Section 5.3 for the response rows pos0 .. pos0 + per - 1 of
+// every batch row, from the attention pass's q, K', masked-input keys and lse.
+struct MassArgs {
+  const void* q;             // [B, Hq, L, 128] bf16
+  const void* k_cached;      // [B, Hkv, L, 128] bf16 (K')
+  const void* k_seedmask;    // [B, Hkv, S, 128] bf16
+  const int32_t* seed_idx;   // [B, S]
+  int n_seeds;
+  const float* lse;          // [B, Hq, L] natural-log lse of the attention pass
+  int B, Hq, Hkv, L, pos0, per;
+  const int32_t* tok;        // [B * per] updated tokens
+  const uint8_t* flags;      // [B * per] bit 1: drafted in this step
+  int mask_id;
+  void* workspace;           // mass_workspace_bytes(B, Hq, per)
+  float* d_in;               // [B * per]
+  float* d_out;              // [B * per]
+};
+size_t mass_workspace_bytes(int B, int Hq, int per);
+int launch_attn_mass(const MassArgs& a, int* status, cudaStream_t stream);
 
 // Seed K/V cache (Section 5.1): gather (override_swap = false) or the override
 // swap (true) of rows of row_bytes (a multiple of 16) bytes.

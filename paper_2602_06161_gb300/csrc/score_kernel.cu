@@ -336,20 +336,20 @@ __device__ __forceinline__ void top_rounds(const uint64_t* keys, int n, int k, u
   __syncthreads();
 }
 
-// The last CTA of a segment: one decoding step's decisions for that sequence.
+// Sections 5.2 and 3, run by the last CTA of a segment: drafting and the
+// revision of the previous seeds. Updates tok, remask_cnt, flags (bit 1 marks
+// the rows drafted in this step; a drafted row loses bit 0) and ws_u (the
+// uncertainty of each row's updated token: ln Z for drafted and replaced rows).
 // Rows written by other CTAs are read through L2 (__ldcg). The drafting sort
-// runs only when more rows pass the threshold than the budget allows; the
-// selection sort only when seeds are to be chosen.
-__device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n, const ScoreParams& P) {
+// runs only when more rows pass the threshold than the budget allows.
+__device__ void segment_update(uint64_t* keys, int seg, int per_seq, int sort_n, const ScoreParams& P) {
   __shared__ unsigned long long s_fallback;
   __shared__ int s_ri[32];
-  __shared__ int s_cnt[4][32];
-  __shared__ double s_rd[32];
+  __shared__ int s_cnt[3][32];
   __shared__ unsigned long long s_top[2][32];
   __shared__ uint64_t s_sel[kRoundsMax];
   __threadfence();
   const DecideArgs& d = P.dec;
-  float* sscore = reinterpret_cast<float*>(keys + sort_n);   // per-row seed score
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5, nw = nt >> 5;
   const int base = seg * per_seq;
   if (tid == 0) s_fallback = ~0ull;
@@ -396,96 +396,125 @@ __device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n,
       // a drafted row takes its greedy token, whose uncertainty is ln Z
       d.tok[n] = __ldcg(P.argmax + n);
       d.ws_u[n] = __ldcg(d.ws_lnz + n);
-      d.flags[n] = static_cast<uint8_t>(d.flags[n] & ~1u);
+      d.flags[n] = static_cast<uint8_t>((d.flags[n] & ~1u) | 2u);
     }
     __syncthreads();
   }
   if (fallback) n_drafted = 1;
 
-  // Section 5.2 revision of the previous seeds, Section 3 state update, Section 5.3 seed score
-  int kept = 0, replaced = 0, remasked = 0, n_t = 0;
-  double total = 0.0;
-  for (int i = tid; i < sort_n; i += nt) {
-    uint64_t key = 0;
-    if (i < per_seq) {
-      const int n = base + i;
-      int y = d.tok[n];
-      uint8_t fl = d.flags[n];
-      int rc = d.remask_cnt[n];
-      float u;
-      if (all_cand && y == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0) &&
-          __ldcg(P.maxprob + n) > d.tau) {
-        // drafted (every candidate fits the budget)
-        y = __ldcg(P.argmax + n);
-        u = __ldcg(d.ws_lnz + n);
-        fl = static_cast<uint8_t>(fl & ~1u);
-        d.tok[n] = y;
+  // Section 5.2 revision of the previous seeds, Section 3 state update
+  int kept = 0, replaced = 0, remasked = 0;
+  for (int i = tid; i < per_seq; i += nt) {
+    const int n = base + i;
+    const int y = d.tok[n];
+    const uint8_t fl = d.flags[n];
+    if (all_cand && y == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0) &&
+        __ldcg(P.maxprob + n) > d.tau) {
+      // drafted (every candidate fits the budget)
+      d.tok[n] = __ldcg(P.argmax + n);
+      d.ws_u[n] = __ldcg(d.ws_lnz + n);
+      d.flags[n] = static_cast<uint8_t>((fl & ~1u) | 2u);
+    } else if ((fl & 1u) != 0 && y != d.mask_id) {
+      const int yh = __ldcg(P.argmax + n);
+      if (yh == y) {
+        ++kept;
+      } else if (__ldcg(P.maxprob + n) > d.tau) {
+        ++replaced;
+        d.tok[n] = yh;
+        d.ws_u[n] = __ldcg(d.ws_lnz + n);
       } else {
-        u = __ldcg(d.ws_u + n);
+        ++remasked;
+        d.tok[n] = d.mask_id;
+        d.remask_cnt[n] = static_cast<uint8_t>(min(d.remask_cnt[n] + 1, 255));
       }
-      const bool was_seed = (fl & 1u) != 0 && y != d.mask_id;
-      if (was_seed) {
-        const int yh = __ldcg(P.argmax + n);
-        if (yh == y) {
-          ++kept;
-        } else if (__ldcg(P.maxprob + n) > d.tau) {
-          ++replaced;
-          y = yh;
-          u = __ldcg(d.ws_lnz + n);
-        } else {
-          ++remasked;
-          y = d.mask_id;
-          rc = min(rc + 1, 255);
-        }
-        d.tok[n] = y;
-        d.remask_cnt[n] = static_cast<uint8_t>(rc);
-      }
-      d.flags[n] = static_cast<uint8_t>(fl & ~1u);
-      float s = -INFINITY;
-      if (y != d.mask_id) {
-        const float din = P.d_in != nullptr ? P.d_in[n] : 0.0f;
-        const float dout = P.d_out != nullptr ? P.d_out[n] : 0.0f;
-        const float sc = u * (1.0f + din) / (1.0f + dout);
-        if (isfinite(sc)) {
-          s = sc;
-          ++n_t;
-          total += static_cast<double>(sc);
-          if (!was_seed && rc < d.remask_budget) key = rank_key(sc, i);
-        }
-      }
-      P.score[n] = s;
-      sscore[i] = s;
     }
-    keys[i] = key;
   }
-  // one reduction for the four counts and the score sum
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     kept += __shfl_xor_sync(0xffffffffu, kept, o);
     replaced += __shfl_xor_sync(0xffffffffu, replaced, o);
     remasked += __shfl_xor_sync(0xffffffffu, remasked, o);
-    n_t += __shfl_xor_sync(0xffffffffu, n_t, o);
-    total += __shfl_xor_sync(0xffffffffu, total, o);
   }
   if (lane == 0) {
     s_cnt[0][warp] = kept;
     s_cnt[1][warp] = replaced;
     s_cnt[2][warp] = remasked;
-    s_cnt[3][warp] = n_t;
+  }
+  __syncthreads();
+  if (tid == 0 && d.stats != nullptr) {
+    kept = replaced = remasked = 0;
+    for (int w = 0; w < nw; ++w) {
+      kept += s_cnt[0][w];
+      replaced += s_cnt[1][w];
+      remasked += s_cnt[2][w];
+    }
+    int32_t* st = d.stats + static_cast<size_t>(seg) * kDecideStats;
+    st[0] = n_drafted;
+    st[1] = kept;
+    st[2] = replaced;
+    st[3] = remasked;
+  }
+}
+
+// Section 5.3 on the updated state of one segment (all threads of the CTA):
+// seed score of every unmasked row, the adaptive revision rate, and the
+// selection among rows that were not previous seeds and have ReMasks left.
+// Clears flag bits 0 and 1 everywhere, then sets bit 0 on the new seeds.
+// keys: sort_n 64-bit slots of shared memory followed by sort_n floats.
+__device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n, const DecideArgs& d,
+                               const float* d_in, const float* d_out, float* score) {
+  __shared__ int s_ri[32];
+  __shared__ int s_nt[32];
+  __shared__ double s_rd[32];
+  __shared__ unsigned long long s_top[2][32];
+  __shared__ uint64_t s_sel[kRoundsMax];
+  const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5, nw = nt >> 5;
+  const int base = seg * per_seq;
+  float* sscore = reinterpret_cast<float*>(keys + sort_n);   // per-row seed score
+
+  int n_t = 0;
+  double total = 0.0;
+  for (int i = tid; i < sort_n; i += nt) {
+    uint64_t key = 0;
+    if (i < per_seq) {
+      const int n = base + i;
+      const uint8_t fl = d.flags[n];
+      float s = -INFINITY;
+      if (d.tok[n] != d.mask_id) {
+        const float din = d_in != nullptr ? d_in[n] : 0.0f;
+        const float dout = d_out != nullptr ? d_out[n] : 0.0f;
+        const float sc = __ldcg(d.ws_u + n) * (1.0f + din) / (1.0f + dout);
+        if (isfinite(sc)) {
+          s = sc;
+          ++n_t;
+          total += static_cast<double>(sc);
+          if ((fl & 1u) == 0 && d.remask_cnt[n] < d.remask_budget) key = rank_key(sc, i);
+        }
+      }
+      score[n] = s;
+      sscore[i] = s;
+      d.flags[n] = static_cast<uint8_t>(fl & ~3u);
+    }
+    keys[i] = key;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    n_t += __shfl_xor_sync(0xffffffffu, n_t, o);
+    total += __shfl_xor_sync(0xffffffffu, total, o);
+  }
+  if (lane == 0) {
+    s_nt[warp] = n_t;
     s_rd[warp] = total;
   }
   __syncthreads();
-  kept = replaced = remasked = n_t = 0;
+  n_t = 0;
   total = 0.0;
   for (int w = 0; w < nw; ++w) {
-    kept += s_cnt[0][w];
-    replaced += s_cnt[1][w];
-    remasked += s_cnt[2][w];
-    n_t += s_cnt[3][w];
+    n_t += s_nt[w];
     total += s_rd[w];
   }
 
-  // Section 5.3 adaptive revision rate: n_t pi_t = #{ s_j > mean } = #{ n_t s_j > sum s }
+  // adaptive revision rate: n_t pi_t = #{ s_j > mean } = #{ n_t s_j > sum s }
   int above = 0;
   for (int i = tid; i < per_seq; i += nt) {
     const float s = sscore[i];
@@ -496,7 +525,7 @@ __device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n,
   while (k * k < above) ++k;   // ceil(sqrt(n_t pi_t))
   k = min(k, d.max_seeds);
 
-  // selection: the k best eligible rows (keys written above)
+  // the k best eligible rows (keys written above)
   const uint64_t* best = keys;
   if (k > 0 && k <= kRoundsMax) {
     top_rounds(keys, sort_n, k, s_sel, s_top);
@@ -520,13 +549,19 @@ __device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n,
     d.n_seeds[seg] = chosen;
     if (d.stats != nullptr) {
       int32_t* st = d.stats + static_cast<size_t>(seg) * kDecideStats;
-      st[0] = n_drafted;
-      st[1] = kept;
-      st[2] = replaced;
-      st[3] = remasked;
       st[4] = n_t;
       st[5] = above;
     }
+  }
+}
+
+// The last CTA of a segment in decision mode: the update, then (unless only the
+// update was asked for) the selection with the caller's d_in / d_out.
+__device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n, const ScoreParams& P) {
+  segment_update(keys, seg, per_seq, sort_n, P);
+  if (P.dec.phase == 0) {
+    __syncthreads();
+    segment_select(keys, seg, per_seq, sort_n, P.dec, P.d_in, P.d_out, P.score);
   }
 }
 
@@ -759,6 +794,16 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
   }
 }
 
+// Section 5.3 selection as its own launch (one CTA per segment), after the
+// update phase and the d_in / d_out pass.
+constexpr int kSelectThreads = 512;
+__global__ void __launch_bounds__(kSelectThreads) seed_select_kernel(const DecideArgs d, const float* d_in,
+                                                                    const float* d_out, float* score, int per_seq,
+                                                                    int sort_n) {
+  extern __shared__ uint64_t sel_keys[];
+  segment_select(sel_keys, blockIdx.x, per_seq, sort_n, d, d_in, d_out, score);
+}
+
 }  // namespace
 
 namespace {
@@ -798,6 +843,16 @@ int launch_score(const ScoreArgs& a, int* status, cudaStream_t stream) {
 
 int launch_score_decide(const ScoreArgs& a, const DecideArgs& d, int* status, cudaStream_t stream) {
   return launch_score_impl(a, &d, status, stream);
+}
+
+int launch_seed_select(int N, int n_seq, const DecideArgs& d, const float* d_in, const float* d_out, float* score,
+                       cudaStream_t stream) {
+  const int per = N / n_seq;
+  int sort_n = 1;
+  while (sort_n < per) sort_n <<= 1;
+  const size_t smem = (sizeof(uint64_t) + sizeof(float)) * static_cast<size_t>(sort_n);
+  seed_select_kernel<<<n_seq, kSelectThreads, smem, stream>>>(d, d_in, d_out, score, per, sort_n);
+  return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
 
 // ---------------------------------------------------------------------------

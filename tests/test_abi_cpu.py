@@ -104,7 +104,7 @@ def test_workspace_bytes(lib):
 
 def decide(lib, **kw):
     a = dict(logits=P, N=8, V=32, n_seq=2, d_in=None, d_out=None, draft_ok=None, tau=0.8, budget=2, remask_budget=3,
-             mask_id=31, min_one=1, pos0=0, max_seeds=4, tok=P, flags=P, remask_cnt=P, maxprob=P, entropy=P,
+             mask_id=31, min_one=1, pos0=0, max_seeds=4, phase=0, tok=P, flags=P, remask_cnt=P, maxprob=P, entropy=P,
              argmax=P, score=P, seed_idx=P, n_seeds=P, stats=None, workspace=P)
     a.update(kw)
     return lib.cover_score_decide_fwd(*a.values(), None)
@@ -114,7 +114,7 @@ def decide(lib, **kw):
     dict(logits=None), dict(tok=None), dict(flags=None), dict(remask_cnt=None), dict(n_seeds=None),
     dict(workspace=None), dict(N=0), dict(V=0), dict(n_seq=3), dict(N=8194, n_seq=2), dict(budget=-1),
     dict(remask_budget=-1), dict(max_seeds=-1), dict(seed_idx=None), dict(logits=P + 2), dict(workspace=P + 4),
-    dict(tok=P + 2),
+    dict(tok=P + 2), dict(phase=2), dict(phase=-1),
 ])
 def test_decide_invalid_args(lib, kw):
     assert decide(lib, **kw) == -1
@@ -157,3 +157,30 @@ def test_prefix_invalid_args(lib, fn, kw):
 
 def test_prefix_unsupported_head_dim(lib):
     assert lib.cover_attn_fwd_prefix(P, P, P, P, P, P, 4, 1, 4, 2, 50, 100, 50, 64, P, None, None) == -2
+
+
+@pytest.mark.parametrize("kw", [
+    dict(tok=None), dict(flags=None), dict(rc=None), dict(score=None), dict(n_seeds=None), dict(ws=None),
+    dict(N=0), dict(n_seq=3), dict(N=8194, n_seq=2), dict(remask_budget=-1), dict(max_seeds=-1),
+    dict(seed_idx=None), dict(ws=P + 4),
+])
+def test_select_invalid_args(lib, kw):
+    a = dict(N=8, n_seq=2, d_in=None, d_out=None, remask_budget=3, mask_id=31, pos0=0, max_seeds=4, tok=P, flags=P,
+             rc=P, score=P, seed_idx=P, n_seeds=P, stats=None, ws=P)
+    a.update(kw)
+    assert lib.cover_seed_select_fwd(*a.values(), None) == -1
+
+
+@pytest.mark.parametrize("kw", [
+    dict(q=None), dict(lse=None), dict(tok=None), dict(ws=None), dict(d_in=None), dict(B=0), dict(Hq=3),
+    dict(per=0), dict(pos0=-1), dict(pos0=10, per=7), dict(n_seeds=17), dict(seed_idx=None), dict(q=P + 8),
+])
+def test_mass_invalid_args(lib, kw):
+    a = dict(q=P, k=P, km=P, seed_idx=P, n_seeds=2, lse=P, B=1, Hq=4, Hkv=2, L=16, D=128, tok=P, flags=P,
+             mask_id=9, pos0=8, per=8, ws=P, d_in=P, d_out=P)
+    a.update(kw)
+    assert lib.cover_attn_mass_fwd(*a.values(), None) == -1
+
+
+def test_mass_unsupported_head_dim(lib):
+    assert lib.cover_attn_mass_fwd(P, P, P, P, 2, P, 1, 4, 2, 16, 64, P, P, 9, 8, 8, P, P, P, None) == -2
