@@ -18,6 +18,8 @@ Printed JSON line (rank 0):
   seed_kv      per-layer seed K/V cache gather and override swap
   prefix_window  the attention of the last block's query rows over the full
                memory (prefix-cache decoding)
+  mass         the decision step in Section 5.3's order: update, d_in / d_out
+               of the response block from the attention pass, selection
   cpu_baseline the fp64 oracle on a bounded sample of the same workload
 
 ``--impl reference`` times the fp64 oracle (the only reference there is: the
@@ -55,7 +57,7 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-secondary", action="store_true")
-    ap.add_argument("--only", choices=["attn", "score", "decide"], default=None,
+    ap.add_argument("--only", choices=["attn", "score", "decide", "mass"], default=None,
                     help="time one kernel alone on the workload (for profiler captures)")
     return ap.parse_args()
 
@@ -352,6 +354,8 @@ def run_ours(args):
         per = {WORKLOAD: seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops)}
         kv_all = {WORKLOAD: kv_timing(api, torch, kc, vc, seeds)}
         prefix_all = {WORKLOAD: prefix_timing(api, torch, q, kc, vc, km, vm, seeds, 64, peak)}
+        api.cover_attn_fwd(q, kc, vc, km, vm, seeds, out=out, lse=lse)   # the seeded pass's lse
+        result["mass"] = mass_timing(api, torch, wl, q, kc, km, seeds, lse)
         del q, kc, vc, km, vm, logits
         torch.cuda.empty_cache()
         scoring_all = {WORKLOAD: scoring["gbs"]}
@@ -473,6 +477,58 @@ def decide_timing(api, torch, wl, iters=20):
             "gbs": round(nbytes / (t_dec * 1e-3) / 1e9, 1),
             "drafted_per_seq": round(float(stats[:, 0].mean()), 2),
             "seeds_per_seq": round(float(out["n_seeds"].float().mean().item()), 2)}
+
+
+def mass_timing(api, torch, wl, q, kc, km, seeds, lse, iters=20):
+    """The three-phase decision step on the workload: update (fused into scoring), d_in / d_out of the
+    response block from the attention pass (`lse` as the attention kernel wrote it), selection."""
+    di = wl.decide_inputs()
+    per = di.N // di.n_seq
+    pos0 = wl.L - per
+    logits = bf16_dev(di.logits, torch)
+    tok0, flags0, rc0 = (torch.from_numpy(x).cuda() for x in (di.tok, di.flags, di.remask_cnt))
+    tok, flags, rc = tok0.clone(), flags0.clone(), rc0.clone()
+    ws = api.decide_workspace(di.N, di.n_seq)
+    mws = torch.empty((api.cover_attn_mass_workspace_bytes(wl.B, wl.Hq, per) + 15) // 16, 4, dtype=torch.int32,
+                      device="cuda")
+    d_in = torch.empty(di.N, dtype=torch.float32, device="cuda")
+    d_out = torch.empty_like(d_in)
+    kw = dict(tau_draft=0.9, draft_budget=15, remask_budget=5, mask_id=di.mask_id, pos0=pos0,
+              max_seeds=wl.score_topk)
+    upd = api.cover_score_decide_fwd(logits, di.n_seq, tok, flags, rc, phase=api.COVER_DECIDE_UPDATE, workspace=ws,
+                                     **kw)
+    sel = api.cover_seed_select_fwd(di.n_seq, tok, flags, rc, ws, remask_budget=5, mask_id=di.mask_id, pos0=pos0,
+                                    max_seeds=wl.score_topk, d_in=d_in, d_out=d_out)
+    stream = torch.cuda.current_stream()
+    phases = {
+        "update": lambda: api.cover_score_decide_fwd(logits, di.n_seq, tok, flags, rc,
+                                                     phase=api.COVER_DECIDE_UPDATE, workspace=ws, out=upd, **kw),
+        "mass": lambda: api.cover_attn_mass_fwd(q, kc, lse, tok, flags, mask_id=di.mask_id, pos0=pos0, per=per,
+                                                k_seedmask=km, seed_idx=seeds, workspace=mws, d_in=d_in,
+                                                d_out=d_out),
+        "select": lambda: api.cover_seed_select_fwd(di.n_seq, tok, flags, rc, ws, remask_budget=5,
+                                                    mask_id=di.mask_id, pos0=pos0, max_seeds=wl.score_topk,
+                                                    d_in=d_in, d_out=d_out, out=sel),
+    }
+    ts = {k: [] for k in phases}
+    for _ in range(iters):
+        tok.copy_(tok0)
+        flags.copy_(flags0)
+        rc.copy_(rc0)
+        for k, fn in phases.items():   # in order: each phase consumes the previous one's state
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            busy_ahead(torch)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts[k].append(a.elapsed_time(b))
+    med = {k: statistics.median(v) for k, v in ts.items()}
+    # tensor work of the mass pass: Q K'^T of the response block, 2 * per^2 * D per head
+    flops = 2.0 * wl.B * wl.Hq * per * per * wl.D
+    return {"response_rows": per, "ms_update": round(med["update"], 4), "ms_mass": round(med["mass"], 4),
+            "ms_select": round(med["select"], 4), "mass_tflops": round(flops / (med["mass"] * 1e-3) / 1e12, 2),
+            "ms_total": round(sum(med.values()), 4)}
 
 
 def prefix_timing(api, torch, q, kc, vc, km, vm, seeds, Lq, peak, iters=20):
@@ -693,6 +749,17 @@ def run_only(args):
         logits = bf16_dev(si.logits, torch)
         wsp = api.score_workspace(si.n_seq)
         fn = lambda: api.cover_score_fwd(logits, si.n_seq, si.topk, workspace=wsp)  # noqa: E731
+    elif args.only == "mass":
+        ai = wl.attn_inputs()
+        q, kc, vc = bf16_dev(ai.q, torch), bf16_dev(ai.k_cached, torch), bf16_dev(ai.v_cached, torch)
+        km, vm = bf16_dev(ai.k_seedmask, torch), bf16_dev(ai.v_seedmask, torch)
+        seeds = torch.from_numpy(ai.seed_idx).cuda()
+        _, lse = api.cover_attn_fwd(q, kc, vc, km, vm, seeds)
+        di = wl.decide_inputs()
+        per = di.N // di.n_seq
+        tok, flags = torch.from_numpy(di.tok).cuda(), torch.from_numpy(di.flags | 2 * di.draft_ok).cuda()
+        fn = lambda: api.cover_attn_mass_fwd(  # noqa: E731
+            q, kc, lse, tok, flags, mask_id=di.mask_id, pos0=wl.L - per, per=per, k_seedmask=km, seed_idx=seeds)
     else:
         di = wl.decide_inputs()
         logits = bf16_dev(di.logits, torch)
