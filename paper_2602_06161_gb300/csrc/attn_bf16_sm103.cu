@@ -116,7 +116,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tail_valid = Lk - (nkv - 1) * kBN;   // valid keys in the last KV tile (1..128)
 
   // ---------------- prologue ----------------
-  if (tid == 0) {
+  // The TMA thread sets up the barriers and issues Q and the first K/V stages at
+  // once, so their latency overlaps tensor-memory allocation and seed routing.
+  const int n_early = min(nkv, kStages);   // K/V stages issued before the CTA-wide barrier
+  if (warp == kTmaWarp && lane == 0) {
     mbar_init(&sm.bar_q, 1);
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.bar_k_full[s], 1);
@@ -132,6 +135,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&sm.bar_drain, 1);
     sm.abort = 0;
     fence_mbar_init();
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_k);
+    tma_prefetch_desc(&tm_v);
+    mbar_arrive_expect_tx(&sm.bar_q, nqt * kTileBytes);
+    for (int t = 0; t < nqt; ++t)
+      for (int h = 0; h < 2; ++h)
+        tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q, 64 * h, row0 + t * kBM, hq, b);
+    for (int j = 0; j < n_early; ++j) {
+      mbar_arrive_expect_tx(&sm.bar_k_full[j], kTileBytes);
+      for (int h = 0; h < 2; ++h)
+        tma_load_4d(sm.k[j] + h * kBoxBytes, &tm_k, &sm.bar_k_full[j], 64 * h, j * kBN, hkv, b);
+      mbar_arrive_expect_tx(&sm.bar_v_full[j], kTileBytes);
+      for (int h = 0; h < 2; ++h)
+        tma_load_4d(sm.v[j] + h * kBoxBytes, &tm_v, &sm.bar_v_full[j], 64 * h, j * kBN, hkv, b);
+    }
   }
   if (warp == kMmaWarp) {
     tmem_alloc(&sm.tmem_base, 512);
@@ -152,16 +170,10 @@ __global__ void __launch_bounds__(kThreads, 1)
    if (warp == kTmaWarp) {
     // ---------------- TMA producer ----------------
     if (lane == 0) {
-      tma_prefetch_desc(&tm_q);
-      tma_prefetch_desc(&tm_k);
-      tma_prefetch_desc(&tm_v);
-      mbar_arrive_expect_tx(&sm.bar_q, nqt * kTileBytes);
-      for (int t = 0; t < nqt; ++t)
-        for (int h = 0; h < 2; ++h)
-          tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q, 64 * h, row0 + t * kBM, hq, b);
-      int last_kj = -1, last_vj = -1;   // last KV tiles whose K / V loads were issued
+      // Q and the first n_early K/V stages were issued in the prologue
+      int last_kj = n_early - 1, last_vj = n_early - 1;   // last KV tiles whose K / V loads were issued
       bool ok = true;
-      for (int j = 0; j < nkv && ok; ++j) {
+      for (int j = n_early; j < nkv && ok; ++j) {
         const int st = j & 1, n = j >> 1;
         if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) {
           ok = false;
