@@ -55,13 +55,17 @@ constexpr int kProducerRegs = 136;
 static_assert(2 * 128 * kSoftmaxRegs + 128 * kProducerRegs <= kThreads * kLaunchRegs, "register split");
 constexpr int kMmaWarp = 8;
 constexpr int kTmaWarp = 9;
+constexpr int kRouteWarp = 10;
+constexpr int kSeedWarp = 11;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct AttnSmem {
   uint8_t q[kNQ][kTileBytes];
   uint8_t k[kStages][kTileBytes];
   uint8_t v[kStages][kTileBytes];
-  uint64_t bar_q;
+  uint64_t bar_q_full[kNQ];
+  uint64_t bar_q_empty[kNQ];       // the unit's last Q.K^T product has read Q tile t (tcgen05.commit)
+  uint64_t bar_q_read[kNQ];        // the seed-score warp is done reading Q tile t
   uint64_t bar_k_full[kStages];
   uint64_t bar_k_empty[kStages];
   uint64_t bar_v_full[kStages];
@@ -69,10 +73,14 @@ struct AttnSmem {
   uint64_t bar_s_full[kNQ];
   uint64_t bar_p_full[kNQ];
   uint64_t bar_o_full[kNQ];
+  uint64_t bar_slot_full[2];       // routing of a unit written (double-buffered by unit parity)
+  uint64_t bar_slot_empty[2];      // a unit's routing and self scores consumed (softmax warps, seed warp)
+  uint64_t bar_sself_full[2];      // a unit's seed self scores written
   uint64_t bar_drain;
   uint32_t tmem_base;
   int abort;
-  int slot[kRowsPerCta];
+  int slot[2][kRowsPerCta];
+  float sself[2][kRowsPerCta];     // s_self = q_i . k_i (log2-scaled) of the unit's seed rows
 };
 
 __device__ __forceinline__ uint32_t col_s(int qt) { return qt * 128u; }
@@ -88,6 +96,20 @@ __device__ __forceinline__ void raise_abort(AttnSmem& sm, int* status, int site)
   sm.abort = 1;
 }
 
+// A work unit is 256 query rows (two Q tiles) of one head (b, hq); the grid is
+// persistent and CTA c takes units c, c + gridDim.x, ... in order.
+struct Unit {
+  int mblk, hq, b;
+};
+
+__device__ __forceinline__ Unit unit_of(int u, int n_mblk, int Hq) {
+  Unit w;
+  w.mblk = u % n_mblk;
+  w.hq = (u / n_mblk) % Hq;
+  w.b = u / (n_mblk * Hq);
+  return w;
+}
+
 // NQ: Q tiles holding query rows (1 for a window of at most 128 rows, else 2).
 // kWindow: query row r sits at memory position q0 + r of an Lk-long memory;
 // otherwise Lq = Lk and q0 = 0 are compile-time facts.
@@ -96,19 +118,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ CUtensorMap tm_v, const __nv_bfloat16* __restrict__ k_seedmask,
                      const __nv_bfloat16* __restrict__ v_seedmask, const int32_t* __restrict__ seed_idx, int n_seeds,
-                     int Hq, int Hkv, int Lq_arg, int Lk, int q0_arg, int n_mblk, float scale_log2,
-                     __nv_bfloat16* __restrict__ out,
-                     float* __restrict__ lse, int* status) {
+                     int Hq, int Hkv, int Lq_arg, int Lk, int q0_arg, int n_mblk, int n_units, float scale_log2,
+                     __nv_bfloat16* __restrict__ out, float* __restrict__ lse, int* status) {
   extern __shared__ uint8_t smem_raw[];
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
-  const int mblk = blockIdx.x % n_mblk;
-  const int hq = (blockIdx.x / n_mblk) % Hq;
-  const int b = blockIdx.x / (n_mblk * Hq);
-  const int hkv = hq / (Hq / Hkv);
-  const int row0 = mblk * kRowsPerCta;
+  const int group = Hq / Hkv;
   const int nkv = (Lk + kBN - 1) / kBN;
   constexpr int nqt = NQ;
   const int Lq = kWindow ? Lq_arg : Lk;
@@ -116,21 +133,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tail_valid = Lk - (nkv - 1) * kBN;   // valid keys in the last KV tile (1..128)
 
   // ---------------- prologue ----------------
-  // The TMA thread sets up the barriers and issues Q and the first K/V stages at
-  // once, so their latency overlaps tensor-memory allocation and seed routing.
-  const int n_early = min(nkv, kStages);   // K/V stages issued before the CTA-wide barrier
   if (warp == kTmaWarp && lane == 0) {
-    mbar_init(&sm.bar_q, 1);
+    for (int t = 0; t < kNQ; ++t) {
+      mbar_init(&sm.bar_q_full[t], 1);
+      mbar_init(&sm.bar_q_empty[t], 1);
+      mbar_init(&sm.bar_q_read[t], 1);
+      mbar_init(&sm.bar_s_full[t], 1);
+      mbar_init(&sm.bar_p_full[t], kBM);
+      mbar_init(&sm.bar_o_full[t], 1);
+    }
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.bar_k_full[s], 1);
       mbar_init(&sm.bar_k_empty[s], 1);
       mbar_init(&sm.bar_v_full[s], 1);
       mbar_init(&sm.bar_v_empty[s], 1);
     }
-    for (int t = 0; t < kNQ; ++t) {
-      mbar_init(&sm.bar_s_full[t], 1);
-      mbar_init(&sm.bar_p_full[t], kBM);
-      mbar_init(&sm.bar_o_full[t], 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.bar_slot_full[s], 32);
+      mbar_init(&sm.bar_slot_empty[s], 4 * nqt + 1);
+      mbar_init(&sm.bar_sself_full[s], 1);
     }
     mbar_init(&sm.bar_drain, 1);
     sm.abort = 0;
@@ -138,103 +159,209 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_k);
     tma_prefetch_desc(&tm_v);
-    mbar_arrive_expect_tx(&sm.bar_q, nqt * kTileBytes);
-    for (int t = 0; t < nqt; ++t)
-      for (int h = 0; h < 2; ++h)
-        tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q, 64 * h, row0 + t * kBM, hq, b);
-    for (int j = 0; j < n_early; ++j) {
-      mbar_arrive_expect_tx(&sm.bar_k_full[j], kTileBytes);
-      for (int h = 0; h < 2; ++h)
-        tma_load_4d(sm.k[j] + h * kBoxBytes, &tm_k, &sm.bar_k_full[j], 64 * h, j * kBN, hkv, b);
-      mbar_arrive_expect_tx(&sm.bar_v_full[j], kTileBytes);
-      for (int h = 0; h < 2; ++h)
-        tma_load_4d(sm.v[j] + h * kBoxBytes, &tm_v, &sm.bar_v_full[j], 64 * h, j * kBN, hkv, b);
-    }
   }
   if (warp == kMmaWarp) {
     tmem_alloc(&sm.tmem_base, 512);
     tmem_relinquish();
   }
-  route_clear(sm.slot, kRowsPerCta, tid, kThreads);
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
-  // query row r of this CTA sits at memory position q0 + row0 + r
-  route_scan(sm.slot, seed_idx + static_cast<size_t>(b) * n_seeds, n_seeds, q0 + row0, kRowsPerCta, Lk, tid,
-             kThreads);
-  __syncthreads();
   const uint32_t tbase = sm.tmem_base;
 
   if (warp >= kMmaWarp) {
    setmaxnreg_dec<kProducerRegs>();
    if (warp == kTmaWarp) {
     // ---------------- TMA producer ----------------
+    // K/V tiles run through the two-stage ring across unit boundaries (G counts the
+    // CTA's KV tiles); Q tile t of a unit is loaded once the previous unit's last
+    // Q.K^T product and the tile's seed self scores are done with it.
     if (lane == 0) {
-      // Q and the first n_early K/V stages were issued in the prologue
-      int last_kj = n_early - 1, last_vj = n_early - 1;   // last KV tiles whose K / V loads were issued
+      int G = 0;
+      int last_kg = -1, last_vg = -1;         // last KV tiles whose K / V loads were issued
+      int last_qit[kNQ] = {-1, -1};           // last units whose Q tiles were issued
       bool ok = true;
-      for (int j = n_early; j < nkv && ok; ++j) {
-        const int st = j & 1, n = j >> 1;
-        if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) {
-          ok = false;
-          break;
+      for (int it = 0, u = blockIdx.x; u < n_units && ok; ++it, u += gridDim.x) {
+        const Unit w = unit_of(u, n_mblk, Hq);
+        const int hkv = w.hq / group;
+        for (int j = 0; j < nkv; ++j, ++G) {
+          const int st = G & 1, n = G >> 1;
+          if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&sm.bar_k_full[st], kTileBytes);
+          for (int h = 0; h < 2; ++h)
+            tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, j * kBN, hkv, w.b);
+          last_kg = G;
+          if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&sm.bar_v_full[st], kTileBytes);
+          for (int h = 0; h < 2; ++h)
+            tma_load_4d(sm.v[st] + h * kBoxBytes, &tm_v, &sm.bar_v_full[st], 64 * h, j * kBN, hkv, w.b);
+          last_vg = G;
+          if (j == 0) {
+            for (int t = 0; t < nqt && ok; ++t) {
+              if (it > 0 && (!mbar_wait(&sm.bar_q_empty[t], (it - 1) & 1, &sm.abort) ||
+                             !mbar_wait(&sm.bar_q_read[t], (it - 1) & 1, &sm.abort))) {
+                ok = false;
+                break;
+              }
+              mbar_arrive_expect_tx(&sm.bar_q_full[t], kTileBytes);
+              for (int h = 0; h < 2; ++h)
+                tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q_full[t], 64 * h,
+                            w.mblk * kRowsPerCta + t * kBM, w.hq, w.b);
+              last_qit[t] = it;
+            }
+            if (!ok) break;
+          }
         }
-        mbar_arrive_expect_tx(&sm.bar_k_full[st], kTileBytes);
-        for (int h = 0; h < 2; ++h)
-          tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, j * kBN, hkv, b);
-        last_kj = j;
-        if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) {
-          ok = false;
-          break;
-        }
-        mbar_arrive_expect_tx(&sm.bar_v_full[st], kTileBytes);
-        for (int h = 0; h < 2; ++h)
-          tma_load_4d(sm.v[st] + h * kBoxBytes, &tm_v, &sm.bar_v_full[st], 64 * h, j * kBN, hkv, b);
-        last_vj = j;
       }
       if (!ok) {
         raise_abort(sm, status, 10);
         // let every copy already issued land before the CTA's shared memory is released
-        mbar_wait(&sm.bar_q, 0, nullptr);
-        for (int jj = max(0, last_kj - 1); jj <= last_kj; ++jj)
-          mbar_wait(&sm.bar_k_full[jj & 1], (jj >> 1) & 1, nullptr);
-        for (int jj = max(0, last_vj - 1); jj <= last_vj; ++jj)
-          mbar_wait(&sm.bar_v_full[jj & 1], (jj >> 1) & 1, nullptr);
+        for (int t = 0; t < nqt; ++t)
+          if (last_qit[t] >= 0) mbar_wait(&sm.bar_q_full[t], last_qit[t] & 1, nullptr);
+        for (int g = max(0, last_kg - 1); g <= last_kg; ++g) mbar_wait(&sm.bar_k_full[g & 1], (g >> 1) & 1, nullptr);
+        for (int g = max(0, last_vg - 1); g <= last_vg; ++g) mbar_wait(&sm.bar_v_full[g & 1], (g >> 1) & 1, nullptr);
       }
     }
-  } else if (warp == kMmaWarp) {
+   } else if (warp == kRouteWarp) {
+    // ---------------- seed routing ----------------
+    // slot[r] of a unit = lowest seed slot naming the unit's row r, written one unit
+    // ahead of the softmax warps into a double buffer.
+    for (int it = 0, u = blockIdx.x; u < n_units; ++it, u += gridDim.x) {
+      const int sb = it & 1;
+      if (it >= 2 && !warp_wait(&sm.bar_slot_empty[sb], ((it >> 1) - 1) & 1, &sm.abort)) {
+        if (lane == 0 && !sm.abort) raise_abort(sm, status, 40);
+        break;
+      }
+      const Unit w = unit_of(u, n_mblk, Hq);
+      route_clear(sm.slot[sb], kRowsPerCta, lane, 32);
+      __syncwarp();
+      // query row r of the unit sits at memory position q0 + mblk * 256 + r
+      route_scan(sm.slot[sb], seed_idx + static_cast<size_t>(w.b) * n_seeds, n_seeds,
+                 q0 + w.mblk * kRowsPerCta, kRowsPerCta, Lk, lane, 32);
+      mbar_arrive(&sm.bar_slot_full[sb]);
+    }
+   } else if (warp == kSeedWarp) {
+    // ---------------- seed self scores ----------------
+    // For each seed row of a unit: s_self = q_i . k_i with the masked-input key (log2-scaled),
+    // one row per warp pass (lane l takes dimensions 4l .. 4l+3), and an L2 prefetch of the
+    // masked-input value row for the epilogue's merge. Runs one unit ahead of the softmax
+    // warps, off their critical path.
+    for (int it = 0, u = blockIdx.x; u < n_units; ++it, u += gridDim.x) {
+      const int sb = it & 1;
+      if (!warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort)) {
+        if (lane == 0 && !sm.abort) raise_abort(sm, status, 50);
+        break;
+      }
+      const Unit w = unit_of(u, n_mblk, Hq);
+      const size_t mbase = (static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds;
+      bool ok = true;
+      for (int t = 0; t < nqt; ++t) {
+        if (!warp_wait(&sm.bar_q_full[t], it & 1, &sm.abort)) {
+          ok = false;
+          break;
+        }
+        // byte offset of this lane's 8 bytes inside a row of the 128-byte-swizzled Q tile
+        const int h = lane >> 4, c8 = (lane & 15) >> 1, half = (lane & 1) * 8;
+        for (int rc = 0; rc < kBM; rc += 32) {
+          const int rr = rc + lane;
+          const int sl = sm.slot[sb][t * kBM + rr];
+          const bool seed_row = sl != kNoSlot && w.mblk * kRowsPerCta + t * kBM + rr < Lq;
+          uint32_t pending = __ballot_sync(0xffffffffu, seed_row);
+          while (pending != 0u) {
+            const int src = __ffs(pending) - 1;
+            pending &= pending - 1u;
+            const int row = rc + src;
+            const size_t mrow = (mbase + __shfl_sync(0xffffffffu, sl, src)) * kD;
+            const uint2 kv = __ldg(reinterpret_cast<const uint2*>(k_seedmask + mrow) + lane);
+            if (lane < 2) prefetch_l2(v_seedmask + mrow + 64 * lane);
+            const uint2 qv = *reinterpret_cast<const uint2*>(sm.q[t] + h * kBoxBytes + row * 128 +
+                                                             ((c8 ^ (row & 7)) * 16) + half);
+            const __nv_bfloat162* qp = reinterpret_cast<const __nv_bfloat162*>(&qv);
+            const __nv_bfloat162* kp = reinterpret_cast<const __nv_bfloat162*>(&kv);
+            const float2 q01 = __bfloat1622float2(qp[0]), q23 = __bfloat1622float2(qp[1]);
+            const float2 k01 = __bfloat1622float2(kp[0]), k23 = __bfloat1622float2(kp[1]);
+            float dot = fmaf(q01.x, k01.x, q01.y * k01.y) + fmaf(q23.x, k23.x, q23.y * k23.y);
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+            if (lane == 0) sm.sself[sb][t * kBM + row] = dot * scale_log2;
+          }
+        }
+        // this warp no longer reads Q tile t of the unit
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.bar_q_read[t]);
+      }
+      if (!ok) {
+        if (lane == 0 && !sm.abort) raise_abort(sm, status, 51);
+        break;
+      }
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&sm.bar_sself_full[sb]);
+        mbar_arrive(&sm.bar_slot_empty[sb]);   // done reading the unit's routing
+      }
+    }
+   } else if (warp == kMmaWarp) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       constexpr uint32_t id_qk = idesc_bf16_f32(kBM, kBN, false, false);
       constexpr uint32_t id_pv = idesc_bf16_f32(kBM, kD, false, true);
-      bool ok = mbar_wait(&sm.bar_q, 0, &sm.abort);
-      tc_fence_after_sync();
       // descriptors of stage / tile 0; the others are one tile (kTileBytes >> 4 units) further
       constexpr uint64_t kTileDesc = kTileBytes >> 4;
       const uint64_t dq0 = sdesc_sw128(smem_u32(sm.q[0]), 16, 1024);
       const uint64_t dk0 = sdesc_sw128(smem_u32(sm.k[0]), 16, 1024);
       const uint64_t dv0 = sdesc_sw128(smem_u32(sm.v[0]), kBoxBytes, 1024);
-      // Per KV tile j: PV(0, j-1), S(0, j), PV(1, j-1), S(1, j). Each wait sits right after a
-      // group of products has been queued, so the tensor pipe works while the thread waits.
-      for (int j = 0; j <= nkv && ok; ++j) {
-        const int st = j & 1, pst = (j - 1) & 1;
-        for (int t = 0; t < nqt; ++t) {
-          if (j > 0) {
-            ok = mbar_wait(&sm.bar_p_full[t], (j - 1) & 1, &sm.abort);
+      // O_t (+)= P_t . V(stage); P from tensor memory, V MN-major from shared memory
+      auto issue_pv = [&](int t, int vst, bool acc) {
+#pragma unroll
+        for (int ks = 0; ks < kBN / 16; ++ks)
+          umma_ts(tbase + col_o(t), tbase + col_s(t) + 8 * ks,
+                  dv0 + vst * kTileDesc + static_cast<uint64_t>((ks * 2048) >> 4), id_pv,
+                  (acc || ks > 0) ? 1u : 0u);
+      };
+      // One stream of steps over the CTA's units. Inside a unit, KV tile j issues
+      // PV(0, j-1), S(0, j), PV(1, j-1), S(1, j); at a unit boundary the previous
+      // unit's last products PV(0), PV(1) go first, then the new unit's S(0, 0),
+      // S(1, 0), so one unit's epilogue overlaps the next unit's first products.
+      // Each wait sits right after a group of products has been queued.
+      int G = 0;
+      bool ok = true;
+      for (int it = 0, u = blockIdx.x; ok; ++it, u += gridDim.x) {
+        if (it > 0) {
+          const int pst = (G - 1) & 1;
+          for (int t = 0; t < nqt; ++t) {
+            ok = mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort);
             if (!ok) break;
             tc_fence_after_sync();
-            // O_t += P_t(j-1) . V(j-1); P from tensor memory, V MN-major from shared memory
-#pragma unroll
-            for (int ks = 0; ks < kBN / 16; ++ks)
-              umma_ts(tbase + col_o(t), tbase + col_s(t) + 8 * ks,
-                      dv0 + pst * kTileDesc + static_cast<uint64_t>((ks * 2048) >> 4), id_pv,
-                      (j > 1 || ks > 0) ? 1u : 0u);
-            if (j == nkv) umma_commit(&sm.bar_o_full[t]);
-            if (t == nqt - 1) umma_commit(&sm.bar_v_empty[pst]);
+            issue_pv(t, pst, nkv > 1);
+            umma_commit(&sm.bar_o_full[t]);
           }
-          if (j < nkv) {
+          if (!ok) break;
+          umma_commit(&sm.bar_v_empty[pst]);
+        }
+        if (u >= n_units) break;
+        for (int j = 0; j < nkv && ok; ++j, ++G) {
+          const int st = G & 1, pst = (G - 1) & 1;
+          for (int t = 0; t < nqt; ++t) {
+            if (j > 0) {
+              ok = mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort);
+              if (!ok) break;
+              tc_fence_after_sync();
+              issue_pv(t, pst, j > 1);
+              if (t == nqt - 1) umma_commit(&sm.bar_v_empty[pst]);
+            }
             if (t == 0) {
-              ok = mbar_wait(&sm.bar_k_full[st], (j >> 1) & 1, &sm.abort);
+              ok = mbar_wait(&sm.bar_k_full[st], (G >> 1) & 1, &sm.abort);
+              if (!ok) break;
+              tc_fence_after_sync();
+            }
+            if (j == 0) {
+              ok = mbar_wait(&sm.bar_q_full[t], it & 1, &sm.abort);
               if (!ok) break;
               tc_fence_after_sync();
             }
@@ -247,9 +374,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             umma_commit(&sm.bar_s_full[t]);
             if (t == nqt - 1) umma_commit(&sm.bar_k_empty[st]);
+            if (j == nkv - 1) umma_commit(&sm.bar_q_empty[t]);
             if (t == 0) {
-              // V(j) feeds the P.V products of the next KV step; it was issued long before
-              ok = mbar_wait(&sm.bar_v_full[st], (j >> 1) & 1, &sm.abort);
+              // V(j) feeds the P.V products of the next step; it was issued long before
+              ok = mbar_wait(&sm.bar_v_full[st], (G >> 1) & 1, &sm.abort);
               if (!ok) break;
             }
           }
@@ -271,135 +399,116 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t trow = tbase + (static_cast<uint32_t>((warp & 3) * 32) << 16);
       const uint32_t s_addr = trow + col_s(qt);
       const uint32_t o_addr = trow + col_o(qt);
-      const int grow = row0 + qt * kBM + r;
-      const int my_slot = sm.slot[qt * kBM + r];
-      const bool is_seed = my_slot != kNoSlot && grow < Lq;
-      // the diagonal of a square launch is column r of KV tile (row0 + qt * 128) / 128; in a
-      // window a warp's 32 consecutive rows meet their diagonals in at most two KV tiles
-      const int diag_j = kWindow ? (q0 + grow) / kBN : (row0 + qt * kBM) / kBN;
-      const int diag_c = kWindow ? (q0 + grow) % kBN : r;
-      const bool warp_seed = __any_sync(0xffffffffu, is_seed);
-      const int dj_lo = kWindow ? __shfl_sync(0xffffffffu, diag_j, 0) : diag_j;
-      const int dj_hi = kWindow ? __shfl_sync(0xffffffffu, diag_j, 31) : diag_j;
-      float m_run = -INFINITY, l_run = 0.0f;
       bool ok = true;
+      // Only what the KV loop needs stays live across it; the unit's coordinates are
+      // recomputed for the epilogue.
+      for (int it = 0; blockIdx.x + it * gridDim.x < n_units && ok; ++it) {
+        const int sb = it & 1;
+        int my_slot;
+        int diag_j, diag_c;
+        {
+          const Unit w = unit_of(blockIdx.x + it * gridDim.x, n_mblk, Hq);
+          const int grow = w.mblk * kRowsPerCta + qt * kBM + r;
+          ok = warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort);
+          if (!ok) break;
+          my_slot = sm.slot[sb][qt * kBM + r];
+          if (grow >= Lq) my_slot = kNoSlot;
+          // the diagonal of a square launch is column r of KV tile (row0 + qt * 128) / 128; in a
+          // window a warp's 32 consecutive rows meet their diagonals in at most two KV tiles
+          diag_j = kWindow ? (q0 + grow) / kBN : (w.mblk * kRowsPerCta + qt * kBM) / kBN;
+          diag_c = kWindow ? (q0 + grow) % kBN : r;
+        }
+        const bool is_seed = my_slot != kNoSlot;
+        const bool warp_seed = __any_sync(0xffffffffu, is_seed);
+        const int dj_lo = kWindow ? __shfl_sync(0xffffffffu, diag_j, 0) : diag_j;
+        const int dj_hi = kWindow ? __shfl_sync(0xffffffffu, diag_j, 31) : diag_j;
+        const int g0 = it * nkv;   // the CTA's KV tiles before this unit
+        float m_run = -INFINITY, l_run = 0.0f;
 
-      // Seed rows: score of the masked-input self pair, s_self = q_i . k_i (log2-scaled),
-      // computed up front so its global loads overlap the first tiles; the value row
-      // is prefetched into L2 for the epilogue.
-      float s_self = 0.0f;
-      const size_t mrow = is_seed ? ((static_cast<size_t>(b) * Hkv + hkv) * n_seeds + my_slot) * kD : 0;
-      if (__any_sync(0xffffffffu, is_seed)) {
-        ok = warp_wait(&sm.bar_q, 0, &sm.abort);
-        if (ok && is_seed) {
-          prefetch_l2(v_seedmask + mrow);
-          prefetch_l2(v_seedmask + mrow + 64);
-          const uint4* kmv = reinterpret_cast<const uint4*>(k_seedmask + mrow);
-          float dot[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        for (int j = 0; j < nkv && ok; ++j) {
+          ok = warp_wait(&sm.bar_s_full[qt], (g0 + j) & 1, &sm.abort);
+          if (!ok) break;
+          tc_fence_after_sync();
+          uint32_t raw[4][32];
 #pragma unroll
-          for (int ch = 0; ch < 16; ++ch) {
-            const int h = ch >> 3, c8 = ch & 7;
-            const uint4 qv =
-                *reinterpret_cast<const uint4*>(sm.q[qt] + h * kBoxBytes + r * 128 + ((c8 ^ (r & 7)) * 16));
-            const uint4 kv = __ldg(kmv + ch);
-            const __nv_bfloat162* qp = reinterpret_cast<const __nv_bfloat162*>(&qv);
-            const __nv_bfloat162* kp = reinterpret_cast<const __nv_bfloat162*>(&kv);
+          for (int c = 0; c < 4; ++c) tmem_ld32(s_addr + 32 * c, raw[c]);
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 qf = __bfloat1622float2(qp[e]);
-              const float2 kf = __bfloat1622float2(kp[e]);
-              dot[e] = fmaf(qf.x, kf.x, dot[e]);
-              dot[e] = fmaf(qf.y, kf.y, dot[e]);
+          for (int c = 0; c < 4; ++c) tmem_ld_wait(raw[c]);
+          float* s = reinterpret_cast<float*>(&raw[0][0]);
+          if (j == nkv - 1 && tail_valid < kBN) {
+#pragma unroll
+            for (int c = 0; c < kBN; ++c)
+              if (c >= tail_valid) s[c] = -INFINITY;
+          }
+          if (warp_seed && (j == dj_lo || j == dj_hi)) {
+            // exclusion of the cached diagonal term of a seed row
+            const bool here = is_seed && j == diag_j;
+#pragma unroll
+            for (int c = 0; c < kBN; ++c)
+              if (here && c == diag_c) s[c] = -INFINITY;
+          }
+          // row maximum: four independent 3-input max chains
+          float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
+#pragma unroll
+          for (int c = 4; c + 8 <= kBN; c += 8) {
+            mx0 = fmax3(mx0, s[c], s[c + 1]);
+            mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
+            mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
+            mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
+          }
+          mx0 = fmax3(mx0, s[kBN - 4], s[kBN - 3]);
+          mx1 = fmax3(mx1, s[kBN - 2], s[kBN - 1]);
+          const float m_tile = fmax3(mx0, mx1, fmaxf(mx2, mx3)) * scale_log2;
+          float alpha = 1.0f;
+          bool rescaled = false;
+          if (m_tile > m_run + kRescaleThreshold) {
+            alpha = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m_tile);
+            m_run = m_tile;
+            rescaled = true;
+          }
+          const float m_use = (m_run == -INFINITY) ? 0.0f : m_run;
+          // p = 2^(s * scale - m) on pairs; four independent partial row sums
+          const uint64_t scale2 = f2_pack(scale_log2, scale_log2);
+          const uint64_t negm2 = f2_pack(-m_use, -m_use);
+          uint64_t acc2[4] = {0, 0, 0, 0};
+          uint32_t packed[64];
+#pragma unroll
+          for (int c = 0; c < 64; ++c) {
+            float t0, t1;
+            f2_unpack(f2_fma(f2_pack(s[2 * c], s[2 * c + 1]), scale2, negm2), t0, t1);
+            const float p0 = ex2_approx(t0);
+            const float p1 = ex2_approx(t1);
+            packed[c] = pack_bf16x2(p0, p1);
+            acc2[c & 3] = f2_add(acc2[c & 3], f2_pack(p0, p1));
+          }
+          float rs[8];
+          f2_unpack(f2_add(acc2[0], acc2[1]), rs[0], rs[1]);
+          f2_unpack(f2_add(acc2[2], acc2[3]), rs[2], rs[3]);
+          const float rowsum = (rs[0] + rs[1]) + (rs[2] + rs[3]);
+          l_run = l_run * alpha + rowsum;
+          tmem_st32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&packed[0]));
+          tmem_st32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&packed[32]));
+          if (j > 0 && __any_sync(0xffffffffu, rescaled)) {
+            // O holds the products of tiles < j (complete: they were issued before S(j))
+#pragma unroll 1
+            for (int c = 0; c < 4; ++c) {
+              uint32_t o[32];
+              tmem_ld32(o_addr + 32 * c, o);
+              tmem_ld_wait(o);
+#pragma unroll
+              for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+              tmem_st32(o_addr + 32 * c, o);
             }
           }
-          s_self = ((dot[0] + dot[1]) + (dot[2] + dot[3])) * scale_log2;
+          tmem_st_wait();
+          tc_fence_before_sync();
+          mbar_arrive(&sm.bar_p_full[qt]);
         }
-      }
-
-      for (int j = 0; j < nkv && ok; ++j) {
-        ok = warp_wait(&sm.bar_s_full[qt], j & 1, &sm.abort);
+        if (ok) ok = warp_wait(&sm.bar_o_full[qt], it & 1, &sm.abort);
         if (!ok) break;
-        tc_fence_after_sync();
-        uint32_t raw[4][32];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32(s_addr + 32 * c, raw[c]);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld_wait(raw[c]);
-        float* s = reinterpret_cast<float*>(&raw[0][0]);
-        if (j == nkv - 1 && tail_valid < kBN) {
-#pragma unroll
-          for (int c = 0; c < kBN; ++c)
-            if (c >= tail_valid) s[c] = -INFINITY;
-        }
-        if (warp_seed && (j == dj_lo || j == dj_hi)) {
-          // exclusion of the cached diagonal term of a seed row
-          const bool here = is_seed && j == diag_j;
-#pragma unroll
-          for (int c = 0; c < kBN; ++c)
-            if (here && c == diag_c) s[c] = -INFINITY;
-        }
-        // row maximum: four independent 3-input max chains
-        float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
-#pragma unroll
-        for (int c = 4; c + 8 <= kBN; c += 8) {
-          mx0 = fmax3(mx0, s[c], s[c + 1]);
-          mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
-          mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
-          mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
-        }
-        mx0 = fmax3(mx0, s[kBN - 4], s[kBN - 3]);
-        mx1 = fmax3(mx1, s[kBN - 2], s[kBN - 1]);
-        const float m_tile = fmax3(mx0, mx1, fmaxf(mx2, mx3)) * scale_log2;
-        float alpha = 1.0f;
-        bool rescaled = false;
-        if (m_tile > m_run + kRescaleThreshold) {
-          alpha = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m_tile);
-          m_run = m_tile;
-          rescaled = true;
-        }
-        const float m_use = (m_run == -INFINITY) ? 0.0f : m_run;
-        // p = 2^(s * scale - m) on pairs; four independent partial row sums
-        const uint64_t scale2 = f2_pack(scale_log2, scale_log2);
-        const uint64_t negm2 = f2_pack(-m_use, -m_use);
-        uint64_t acc2[4] = {0, 0, 0, 0};
-        uint32_t packed[64];
-#pragma unroll
-        for (int c = 0; c < 64; ++c) {
-          float t0, t1;
-          f2_unpack(f2_fma(f2_pack(s[2 * c], s[2 * c + 1]), scale2, negm2), t0, t1);
-          const float p0 = ex2_approx(t0);
-          const float p1 = ex2_approx(t1);
-          packed[c] = pack_bf16x2(p0, p1);
-          acc2[c & 3] = f2_add(acc2[c & 3], f2_pack(p0, p1));
-        }
-        float rs[8];
-        f2_unpack(f2_add(acc2[0], acc2[1]), rs[0], rs[1]);
-        f2_unpack(f2_add(acc2[2], acc2[3]), rs[2], rs[3]);
-        const float rowsum = (rs[0] + rs[1]) + (rs[2] + rs[3]);
-        l_run = l_run * alpha + rowsum;
-        tmem_st32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&packed[0]));
-        tmem_st32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&packed[32]));
-        if (j > 0 && __any_sync(0xffffffffu, rescaled)) {
-          // O holds the products of tiles < j (complete: they were issued before S(j))
-#pragma unroll 1
-          for (int c = 0; c < 4; ++c) {
-            uint32_t o[32];
-            tmem_ld32(o_addr + 32 * c, o);
-            tmem_ld_wait(o);
-#pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-            tmem_st32(o_addr + 32 * c, o);
-          }
-        }
-        tmem_st_wait();
-        tc_fence_before_sync();
-        mbar_arrive(&sm.bar_p_full[qt]);
-      }
-      if (ok) ok = warp_wait(&sm.bar_o_full[qt], 0, &sm.abort);
-      if (ok) ok = warp_wait(&sm.bar_q, 0, &sm.abort);
-      if (!ok) {
-        if (!sm.abort) raise_abort(sm, status, 30 + qt);
-      } else {
+        // ---------------- epilogue of the unit ----------------
+        // O is read into registers before this warpgroup's next P is published, so the
+        // next unit's first P.V product cannot overwrite it early.
         tc_fence_after_sync();
         uint32_t oraw[4][32];
 #pragma unroll
@@ -407,8 +516,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int c = 0; c < 4; ++c) tmem_ld_wait(oraw[c]);
         float* o = reinterpret_cast<float*>(&oraw[0][0]);
+        const Unit w = unit_of(blockIdx.x + it * gridDim.x, n_mblk, Hq);
+        const int grow = w.mblk * kRowsPerCta + qt * kBM + r;
+        if (warp_seed) {
+          ok = warp_wait(&sm.bar_sself_full[sb], (it >> 1) & 1, &sm.abort);
+          if (!ok) break;
+        }
         if (is_seed) {
           // merge the masked-input self term (k_i, v_i) of this seed row
+          const float s_self = sm.sself[sb][qt * kBM + r];
+          const size_t mrow = ((static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds + my_slot) * kD;
           const uint4* vmv = reinterpret_cast<const uint4*>(v_seedmask + mrow);
           const float m2 = fmaxf(m_run, s_self);
           const float a = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m2);
@@ -429,20 +546,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (grow < Lq) {
           const float inv = 1.0f / l_run;
-          uint4* dst = reinterpret_cast<uint4*>(out + ((static_cast<size_t>(b) * Hq + hq) * Lq + grow) * kD);
+          const size_t orow = (static_cast<size_t>(w.b) * Hq + w.hq) * Lq + grow;
+          uint4* dst = reinterpret_cast<uint4*>(out + orow * kD);
 #pragma unroll
           for (int ch = 0; ch < 16; ++ch) {
-            uint4 w;
-            w.x = pack_bf16x2(o[ch * 8 + 0] * inv, o[ch * 8 + 1] * inv);
-            w.y = pack_bf16x2(o[ch * 8 + 2] * inv, o[ch * 8 + 3] * inv);
-            w.z = pack_bf16x2(o[ch * 8 + 4] * inv, o[ch * 8 + 5] * inv);
-            w.w = pack_bf16x2(o[ch * 8 + 6] * inv, o[ch * 8 + 7] * inv);
-            dst[ch] = w;
+            uint4 v;
+            v.x = pack_bf16x2(o[ch * 8 + 0] * inv, o[ch * 8 + 1] * inv);
+            v.y = pack_bf16x2(o[ch * 8 + 2] * inv, o[ch * 8 + 3] * inv);
+            v.z = pack_bf16x2(o[ch * 8 + 4] * inv, o[ch * 8 + 5] * inv);
+            v.w = pack_bf16x2(o[ch * 8 + 6] * inv, o[ch * 8 + 7] * inv);
+            dst[ch] = v;
           }
-          if (lse != nullptr)
-            lse[(static_cast<size_t>(b) * Hq + hq) * Lq + grow] = (m_run + log2f(l_run)) * 0.6931471805599453f;
+          if (lse != nullptr) lse[orow] = (m_run + log2f(l_run)) * 0.6931471805599453f;
         }
+        // the unit's routing and self scores are consumed
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.bar_slot_empty[sb]);
       }
+      if (!ok && !sm.abort) raise_abort(sm, status, 30 + qt);
     }
   }
 
@@ -462,8 +583,18 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
       !make_bf16_map_4d(&tv, a.v_cached, kD, a.L, a.Hkv, a.B, kBN))
     return -3;
   const int n_mblk = (a.Lq + kRowsPerCta - 1) / kRowsPerCta;
-  const long long grid = static_cast<long long>(n_mblk) * a.Hq * a.B;
-  if (grid > 0x7fffffffLL) return -2;
+  const long long n_units = static_cast<long long>(n_mblk) * a.Hq * a.B;
+  static int n_sm = 0;
+  if (n_sm == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n_sm < 1)
+      return -3;
+  }
+  // unit indices advance by the grid size past the last unit: keep them inside int
+  if (n_units > 0x7fffffffLL - n_sm) return -2;
+  // persistent grid: one CTA per SM (1 CTA/SM fits), each looping over units
+  const long long grid = n_units < n_sm ? n_units : n_sm;
   const size_t smem = sizeof(AttnSmem) + 1024;
   static bool attr_set = false;
   if (!attr_set) {
@@ -484,9 +615,8 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
                               : attn_bf16_kernel<2, true>;
   kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
       tq, tk, tv, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
-      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, scale_log2, static_cast<__nv_bfloat16*>(a.out),
-      a.lse,
-      status);
+      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, static_cast<int>(n_units), scale_log2,
+      static_cast<__nv_bfloat16*>(a.out), a.lse, status);
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
 
