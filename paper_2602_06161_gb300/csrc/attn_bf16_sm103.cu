@@ -12,12 +12,16 @@
 // r_i, and a seed row never reads k'_i, v'_i while a non-seed row never reads
 // the masked buffer.
 //
-// Structure (one CTA per 256 query rows of one head, 1 CTA per SM):
+// Structure: a persistent grid of one CTA per SM; a work unit is 256 query
+// rows (two Q tiles of 128) of one head, and CTA c takes units c, c + grid,
+// c + 2 grid, ... The pipelines below run across unit boundaries, so one
+// unit's epilogue overlaps the next unit's loads and first products.
 //   warps 0-3  softmax + epilogue of Q tile 0 (thread = row)
 //   warps 4-7  softmax + epilogue of Q tile 1
 //   warp  8    tensor-memory allocation; lane 0 issues tcgen05.mma
-//   warp  9    lane 0 issues TMA loads (Q once, K/V through a 2-stage ring)
-//   warps 10-11 complete the producer warpgroup (register donors, no work)
+//   warp  9    lane 0 issues TMA loads (Q per unit, K/V through a 2-stage ring)
+//   warp  10   seed routing of the next unit (double-buffered slot table)
+//   warp  11   seed self scores q_i . k_i of the next unit, L2 prefetch of v_i
 // Registers: launched at 168 per thread (12 warps); the producer warpgroup
 // gives back down to 136 and the two softmax warpgroups take 184 each
 // (setmaxnreg), so the 128-column softmax rows stay in registers without
@@ -59,6 +63,20 @@ constexpr int kRouteWarp = 10;
 constexpr int kSeedWarp = 11;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
+// A work unit is 256 query rows (two Q tiles) of one head (b, hq); the grid is
+// persistent and CTA c takes units c, c + gridDim.x, ... in order.
+struct Unit {
+  int mblk, hq, b;
+};
+
+__device__ __forceinline__ Unit unit_of(int u, int n_mblk, int Hq) {
+  Unit w;
+  w.mblk = u % n_mblk;
+  w.hq = (u / n_mblk) % Hq;
+  w.b = u / (n_mblk * Hq);
+  return w;
+}
+
 struct AttnSmem {
   uint8_t q[kNQ][kTileBytes];
   uint8_t k[kStages][kTileBytes];
@@ -70,6 +88,9 @@ struct AttnSmem {
   uint64_t bar_k_empty[kStages];
   uint64_t bar_v_full[kStages];
   uint64_t bar_v_empty[kStages];
+  // a stage whose KV tile ended a unit holds that unit's output until the TMA thread
+  // has stored it: K stage for Q tile 0, V stage for Q tile 1
+  uint64_t bar_ostage_full[kNQ];   // the tile's four softmax warps have staged the unit's output
   uint64_t bar_s_full[kNQ];
   uint64_t bar_p_full[kNQ];
   uint64_t bar_o_full[kNQ];
@@ -80,6 +101,7 @@ struct AttnSmem {
   uint32_t tmem_base;
   int abort;
   int slot[2][kRowsPerCta];
+  Unit unit[2];                    // coordinates of the unit whose routing is in slot[sb]
   float sself[2][kRowsPerCta];     // s_self = q_i . k_i (log2-scaled) of the unit's seed rows
 };
 
@@ -96,27 +118,14 @@ __device__ __forceinline__ void raise_abort(AttnSmem& sm, int* status, int site)
   sm.abort = 1;
 }
 
-// A work unit is 256 query rows (two Q tiles) of one head (b, hq); the grid is
-// persistent and CTA c takes units c, c + gridDim.x, ... in order.
-struct Unit {
-  int mblk, hq, b;
-};
-
-__device__ __forceinline__ Unit unit_of(int u, int n_mblk, int Hq) {
-  Unit w;
-  w.mblk = u % n_mblk;
-  w.hq = (u / n_mblk) % Hq;
-  w.b = u / (n_mblk * Hq);
-  return w;
-}
-
 // NQ: Q tiles holding query rows (1 for a window of at most 128 rows, else 2).
 // kWindow: query row r sits at memory position q0 + r of an Lk-long memory;
 // otherwise Lq = Lk and q0 = 0 are compile-time facts.
 template <int NQ, bool kWindow>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                     const __grid_constant__ CUtensorMap tm_v, const __nv_bfloat16* __restrict__ k_seedmask,
+                     const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
+                     const __nv_bfloat16* __restrict__ k_seedmask,
                      const __nv_bfloat16* __restrict__ v_seedmask, const int32_t* __restrict__ seed_idx, int n_seeds,
                      int Hq, int Hkv, int Lq_arg, int Lk, int q0_arg, int n_mblk, int n_units, float scale_log2,
                      __nv_bfloat16* __restrict__ out, float* __restrict__ lse, int* status) {
@@ -141,6 +150,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sm.bar_s_full[t], 1);
       mbar_init(&sm.bar_p_full[t], kBM);
       mbar_init(&sm.bar_o_full[t], 1);
+      mbar_init(&sm.bar_ostage_full[t], 4);
     }
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.bar_k_full[s], 1);
@@ -159,6 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_k);
     tma_prefetch_desc(&tm_v);
+    tma_prefetch_desc(&tm_o);
   }
   if (warp == kMmaWarp) {
     tmem_alloc(&sm.tmem_base, 512);
@@ -180,13 +191,50 @@ __global__ void __launch_bounds__(kThreads, 1)
       int G = 0;
       int last_kg = -1, last_vg = -1;         // last KV tiles whose K / V loads were issued
       int last_qit[kNQ] = {-1, -1};           // last units whose Q tiles were issued
+      int n_stored = 0;                       // units whose output the thread has stored
       bool ok = true;
+      // Stores unit n's output of Q tile t from the stage its last KV tile used, once the
+      // tile's softmax warps have staged it; returns after the copies have read the stage.
+      auto store_unit = [&](int n, int t) {
+        if (!mbar_wait(&sm.bar_ostage_full[t], n & 1, &sm.abort)) return false;
+        const Unit wn = unit_of(blockIdx.x + n * gridDim.x, n_mblk, Hq);
+        const int sig = (n * nkv + nkv - 1) & 1;
+        const uint8_t* stage = t == 0 ? sm.k[sig] : sm.v[sig];
+        for (int wq = 0; wq < 4; ++wq) {
+          const int wrow = wn.mblk * kRowsPerCta + t * kBM + wq * 32;
+          if (wrow < Lq) {   // rows at or past Lq fall outside the tensor and are not written
+            tma_store_4d(&tm_o, stage + wq * 8192, 0, wrow, wn.hq, wn.b);
+            tma_store_4d(&tm_o, stage + wq * 8192 + 4096, 64, wrow, wn.hq, wn.b);
+          }
+        }
+        bulk_commit_group();
+        bulk_wait_group_read0();
+        return true;
+      };
       for (int it = 0, u = blockIdx.x; u < n_units && ok; ++it, u += gridDim.x) {
         const Unit w = unit_of(u, n_mblk, Hq);
         const int hkv = w.hq / group;
+        // Q tile t of the unit: wait until the previous unit is done with the buffer
+        auto load_q = [&](int t) {
+          if (it > 0 && (!mbar_wait(&sm.bar_q_empty[t], (it - 1) & 1, &sm.abort) ||
+                         !mbar_wait(&sm.bar_q_read[t], (it - 1) & 1, &sm.abort)))
+            return false;
+          mbar_arrive_expect_tx(&sm.bar_q_full[t], kTileBytes);
+          for (int h = 0; h < 2; ++h)
+            tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q_full[t], 64 * h, w.mblk * kRowsPerCta + t * kBM,
+                        w.hq, w.b);
+          last_qit[t] = it;
+          return true;
+        };
         for (int j = 0; j < nkv; ++j, ++G) {
           const int st = G & 1, n = G >> 1;
+          // tile G - 2 (same stage) was the last of a unit: the stage staged that unit's output
+          const bool staged = G >= 2 && (G - 2) % nkv == nkv - 1;
           if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) {
+            ok = false;
+            break;
+          }
+          if (staged && !store_unit(n_stored, 0)) {
             ok = false;
             break;
           }
@@ -194,31 +242,44 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int h = 0; h < 2; ++h)
             tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, j * kBN, hkv, w.b);
           last_kg = G;
+          if (j == 0 && !load_q(0)) {
+            ok = false;
+            break;
+          }
           if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) {
             ok = false;
             break;
+          }
+          if (staged) {
+            if (nqt > 1 && !store_unit(n_stored, 1)) {
+              ok = false;
+              break;
+            }
+            ++n_stored;
           }
           mbar_arrive_expect_tx(&sm.bar_v_full[st], kTileBytes);
           for (int h = 0; h < 2; ++h)
             tma_load_4d(sm.v[st] + h * kBoxBytes, &tm_v, &sm.bar_v_full[st], 64 * h, j * kBN, hkv, w.b);
           last_vg = G;
           if (j == 0) {
-            for (int t = 0; t < nqt && ok; ++t) {
-              if (it > 0 && (!mbar_wait(&sm.bar_q_empty[t], (it - 1) & 1, &sm.abort) ||
-                             !mbar_wait(&sm.bar_q_read[t], (it - 1) & 1, &sm.abort))) {
-                ok = false;
-                break;
-              }
-              mbar_arrive_expect_tx(&sm.bar_q_full[t], kTileBytes);
-              for (int h = 0; h < 2; ++h)
-                tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q_full[t], 64 * h,
-                            w.mblk * kRowsPerCta + t * kBM, w.hq, w.b);
-              last_qit[t] = it;
-            }
+            for (int t = 1; t < nqt && ok; ++t) ok = load_q(t);
             if (!ok) break;
+            // the next unit's Q tiles go to L2 now, so their loads at the boundary are short
+            if (u + static_cast<int>(gridDim.x) < n_units) {
+              const Unit wn = unit_of(u + gridDim.x, n_mblk, Hq);
+              for (int t = 0; t < nqt; ++t)
+                for (int h = 0; h < 2; ++h)
+                  tma_prefetch_l2_4d(&tm_q, 64 * h, wn.mblk * kRowsPerCta + t * kBM, wn.hq, wn.b);
+            }
           }
         }
       }
+      // the units whose stages were not needed again
+      const int n_iters = (n_units - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
+                          static_cast<int>(gridDim.x);
+      for (; ok && n_stored < n_iters; ++n_stored)
+        for (int t = 0; t < nqt && ok; ++t) ok = store_unit(n_stored, t);
+      bulk_wait_group0();
       if (!ok) {
         raise_abort(sm, status, 10);
         // let every copy already issued land before the CTA's shared memory is released
@@ -239,6 +300,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       const Unit w = unit_of(u, n_mblk, Hq);
+      if (lane == 0) sm.unit[sb] = w;
       route_clear(sm.slot[sb], kRowsPerCta, lane, 32);
       __syncwarp();
       // query row r of the unit sits at memory position q0 + mblk * 256 + r
@@ -258,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0 && !sm.abort) raise_abort(sm, status, 50);
         break;
       }
-      const Unit w = unit_of(u, n_mblk, Hq);
+      const Unit w = sm.unit[sb];
       const size_t mbase = (static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds;
       bool ok = true;
       for (int t = 0; t < nqt; ++t) {
@@ -407,10 +469,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         int my_slot;
         int diag_j, diag_c;
         {
-          const Unit w = unit_of(blockIdx.x + it * gridDim.x, n_mblk, Hq);
-          const int grow = w.mblk * kRowsPerCta + qt * kBM + r;
           ok = warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort);
           if (!ok) break;
+          const Unit w = sm.unit[sb];
+          const int grow = w.mblk * kRowsPerCta + qt * kBM + r;
           my_slot = sm.slot[sb][qt * kBM + r];
           if (grow >= Lq) my_slot = kNoSlot;
           // the diagonal of a square launch is column r of KV tile (row0 + qt * 128) / 128; in a
@@ -516,7 +578,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int c = 0; c < 4; ++c) tmem_ld_wait(oraw[c]);
         float* o = reinterpret_cast<float*>(&oraw[0][0]);
-        const Unit w = unit_of(blockIdx.x + it * gridDim.x, n_mblk, Hq);
+        const Unit w = sm.unit[sb];
         const int grow = w.mblk * kRowsPerCta + qt * kBM + r;
         if (warp_seed) {
           ok = warp_wait(&sm.bar_sself_full[sb], (it >> 1) & 1, &sm.abort);
@@ -544,10 +606,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           m_run = m2;
         }
-        if (grow < Lq) {
+        // Output: the warp's 32 rows x 128 columns are staged in the shared-memory stage of
+        // the unit's last KV tile (K stage for Q tile 0, V stage for Q tile 1: both finished
+        // with once O is complete) as two 128-byte-swizzled boxes of 64 columns; the TMA
+        // thread writes them out, so the global writes are full lines instead of one 16-byte
+        // piece per row, and this warp goes on to the next unit at once.
+        {
+          const int sig = (g0 + nkv - 1) & 1;
+          uint8_t* stage = (qt == 0 ? sm.k[sig] : sm.v[sig]) + (warp & 3) * (2 * 4096);
           const float inv = 1.0f / l_run;
-          const size_t orow = (static_cast<size_t>(w.b) * Hq + w.hq) * Lq + grow;
-          uint4* dst = reinterpret_cast<uint4*>(out + orow * kD);
 #pragma unroll
           for (int ch = 0; ch < 16; ++ch) {
             uint4 v;
@@ -555,9 +622,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             v.y = pack_bf16x2(o[ch * 8 + 2] * inv, o[ch * 8 + 3] * inv);
             v.z = pack_bf16x2(o[ch * 8 + 4] * inv, o[ch * 8 + 5] * inv);
             v.w = pack_bf16x2(o[ch * 8 + 6] * inv, o[ch * 8 + 7] * inv);
-            dst[ch] = v;
+            *reinterpret_cast<uint4*>(stage + (ch >> 3) * 4096 + lane * 128 + (((ch & 7) ^ (lane & 7)) << 4)) = v;
           }
-          if (lse != nullptr) lse[orow] = (m_run + log2f(l_run)) * 0.6931471805599453f;
+          if (lse != nullptr && grow < Lq)
+            lse[(static_cast<size_t>(w.b) * Hq + w.hq) * Lq + grow] = (m_run + log2f(l_run)) * 0.6931471805599453f;
+          // the staged rows go to the TMA thread, which stores them before it reloads the stage
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.bar_ostage_full[qt]);
         }
         // the unit's routing and self scores are consumed
         __syncwarp();
@@ -577,8 +649,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace
 
 int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) {
-  CUtensorMap tq, tk, tv;
+  CUtensorMap tq, tk, tv, to;
   if (!make_bf16_map_4d(&tq, a.q, kD, a.Lq, a.Hq, a.B, kBM) ||
+      !make_bf16_map_4d(&to, a.out, kD, a.Lq, a.Hq, a.B, 32) ||
       !make_bf16_map_4d(&tk, a.k_cached, kD, a.L, a.Hkv, a.B, kBN) ||
       !make_bf16_map_4d(&tv, a.v_cached, kD, a.L, a.Hkv, a.B, kBN))
     return -3;
@@ -614,7 +687,7 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
                 : a.Lq <= kBM ? attn_bf16_kernel<1, true>
                               : attn_bf16_kernel<2, true>;
   kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
-      tq, tk, tv, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
+      tq, tk, tv, to, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
       a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, static_cast<int>(n_units), scale_log2,
       static_cast<__nv_bfloat16*>(a.out), a.lse, status);
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
