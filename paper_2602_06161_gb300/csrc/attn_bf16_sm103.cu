@@ -108,6 +108,14 @@ struct AttnSmem {
 __device__ __forceinline__ uint32_t col_s(int qt) { return qt * 128u; }
 __device__ __forceinline__ uint32_t col_o(int qt) { return 256u + qt * 128u; }
 
+// Sets s[32 * K + i] to -inf where bit i of sel is set (K a compile-time chunk index).
+template <int K>
+__device__ __forceinline__ void exclude_in_chunk(float* s, uint32_t sel) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i)
+    if ((sel >> i) & 1u) s[32 * K + i] = -INFINITY;
+}
+
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
   const bool ok = mbar_wait(bar, parity, abort);
   return __all_sync(0xffffffffu, ok);
@@ -505,9 +513,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (warp_seed && (j == dj_lo || j == dj_hi)) {
             // exclusion of the cached diagonal term of a seed row
             const bool here = is_seed && j == diag_j;
+            if (!kWindow) {
+              // square launch: row r's diagonal is column r, element `lane` of 32-column chunk warp & 3
+              const uint32_t sel = here ? (1u << lane) : 0u;
+              switch (warp & 3) {
+                case 0: exclude_in_chunk<0>(s, sel); break;
+                case 1: exclude_in_chunk<1>(s, sel); break;
+                case 2: exclude_in_chunk<2>(s, sel); break;
+                default: exclude_in_chunk<3>(s, sel); break;
+              }
+            } else {
 #pragma unroll
-            for (int c = 0; c < kBN; ++c)
-              if (here && c == diag_c) s[c] = -INFINITY;
+              for (int c = 0; c < kBN; ++c)
+                if (here && c == diag_c) s[c] = -INFINITY;
+            }
           }
           // row maximum: four independent 3-input max chains
           float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
