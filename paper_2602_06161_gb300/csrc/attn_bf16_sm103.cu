@@ -62,6 +62,8 @@ constexpr int kTmaWarp = 9;
 constexpr int kRouteWarp = 10;
 constexpr int kSeedWarp = 11;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+constexpr int kVStageRows = 32;            // masked value rows of a unit staged in shared memory
+constexpr int kNotStaged = 255;
 
 // A work unit is 256 query rows (two Q tiles) of one head (b, hq); the grid is
 // persistent and CTA c takes units c, c + gridDim.x, ... in order.
@@ -103,6 +105,8 @@ struct AttnSmem {
   int slot[2][kRowsPerCta];
   Unit unit[2];                    // coordinates of the unit whose routing is in slot[sb]
   float sself[2][kRowsPerCta];     // s_self = q_i . k_i (log2-scaled) of the unit's seed rows
+  uint8_t vidx[2][kRowsPerCta];    // a seed row's staged value row, or kNotStaged
+  alignas(16) uint8_t vstage[2][kVStageRows][kD * 2];   // masked-input value rows v_i, bf16
 };
 
 __device__ __forceinline__ uint32_t col_s(int qt) { return qt * 128u; }
@@ -319,9 +323,10 @@ __global__ void __launch_bounds__(kThreads, 1)
    } else if (warp == kSeedWarp) {
     // ---------------- seed self scores ----------------
     // For each seed row of a unit: s_self = q_i . k_i with the masked-input key (log2-scaled),
-    // one row per warp pass (lane l takes dimensions 4l .. 4l+3), and an L2 prefetch of the
-    // masked-input value row for the epilogue's merge. Runs one unit ahead of the softmax
-    // warps, off their critical path.
+    // one row per warp pass (lane l takes dimensions 4l .. 4l+3), and the masked-input value
+    // row v_i copied into shared memory for the epilogue's merge (the unit's first 32 seed
+    // rows; the epilogue reads any others from global memory). Runs one unit ahead of the
+    // softmax warps, off their critical path.
     for (int it = 0, u = blockIdx.x; u < n_units; ++it, u += gridDim.x) {
       const int sb = it & 1;
       if (!warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort)) {
@@ -330,6 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const Unit w = sm.unit[sb];
       const size_t mbase = (static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds;
+      int n_staged = 0;
       bool ok = true;
       for (int t = 0; t < nqt; ++t) {
         if (!warp_wait(&sm.bar_q_full[t], it & 1, &sm.abort)) {
@@ -344,22 +350,41 @@ __global__ void __launch_bounds__(kThreads, 1)
           const bool seed_row = sl != kNoSlot && w.mblk * kRowsPerCta + t * kBM + rr < Lq;
           uint32_t pending = __ballot_sync(0xffffffffu, seed_row);
           while (pending != 0u) {
-            const int src = __ffs(pending) - 1;
-            pending &= pending - 1u;
-            const int row = rc + src;
-            const size_t mrow = (mbase + __shfl_sync(0xffffffffu, sl, src)) * kD;
-            const uint2 kv = __ldg(reinterpret_cast<const uint2*>(k_seedmask + mrow) + lane);
-            if (lane < 2) prefetch_l2(v_seedmask + mrow + 64 * lane);
-            const uint2 qv = *reinterpret_cast<const uint2*>(sm.q[t] + h * kBoxBytes + row * 128 +
-                                                             ((c8 ^ (row & 7)) * 16) + half);
-            const __nv_bfloat162* qp = reinterpret_cast<const __nv_bfloat162*>(&qv);
-            const __nv_bfloat162* kp = reinterpret_cast<const __nv_bfloat162*>(&kv);
-            const float2 q01 = __bfloat1622float2(qp[0]), q23 = __bfloat1622float2(qp[1]);
-            const float2 k01 = __bfloat1622float2(kp[0]), k23 = __bfloat1622float2(kp[1]);
-            float dot = fmaf(q01.x, k01.x, q01.y * k01.y) + fmaf(q23.x, k23.x, q23.y * k23.y);
+            // up to four seed rows at a time, their loads in flight together
+            int row[4];
+            uint2 kv[4], vv[4];
 #pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
-            if (lane == 0) sm.sself[sb][t * kBM + row] = dot * scale_log2;
+            for (int g = 0; g < 4; ++g) {
+              row[g] = -1;
+              if (pending != 0u) {
+                const int src = __ffs(pending) - 1;
+                pending &= pending - 1u;
+                row[g] = rc + src;
+                const size_t mrow = (mbase + __shfl_sync(0xffffffffu, sl, src)) * kD;
+                kv[g] = __ldg(reinterpret_cast<const uint2*>(k_seedmask + mrow) + lane);
+                vv[g] = __ldg(reinterpret_cast<const uint2*>(v_seedmask + mrow) + lane);
+              }
+            }
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+              if (row[g] < 0) continue;
+              const uint2 qv = *reinterpret_cast<const uint2*>(sm.q[t] + h * kBoxBytes + row[g] * 128 +
+                                                               ((c8 ^ (row[g] & 7)) * 16) + half);
+              const __nv_bfloat162* qp = reinterpret_cast<const __nv_bfloat162*>(&qv);
+              const __nv_bfloat162* kp = reinterpret_cast<const __nv_bfloat162*>(&kv[g]);
+              const float2 q01 = __bfloat1622float2(qp[0]), q23 = __bfloat1622float2(qp[1]);
+              const float2 k01 = __bfloat1622float2(kp[0]), k23 = __bfloat1622float2(kp[1]);
+              float dot = fmaf(q01.x, k01.x, q01.y * k01.y) + fmaf(q23.x, k23.x, q23.y * k23.y);
+#pragma unroll
+              for (int o = 16; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+              // the first kVStageRows seed rows of the unit keep v_i in shared memory
+              const int vi = n_staged < kVStageRows ? n_staged++ : kNotStaged;
+              if (vi != kNotStaged) reinterpret_cast<uint2*>(sm.vstage[sb][vi])[lane] = vv[g];
+              if (lane == 0) {
+                sm.sself[sb][t * kBM + row[g]] = dot * scale_log2;
+                sm.vidx[sb][t * kBM + row[g]] = static_cast<uint8_t>(vi);
+              }
+            }
           }
         }
         // this warp no longer reads Q tile t of the unit
@@ -606,15 +631,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (is_seed) {
           // merge the masked-input self term (k_i, v_i) of this seed row
           const float s_self = sm.sself[sb][qt * kBM + r];
+          const int vi = sm.vidx[sb][qt * kBM + r];
           const size_t mrow = ((static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds + my_slot) * kD;
-          const uint4* vmv = reinterpret_cast<const uint4*>(v_seedmask + mrow);
+          // generic loads: shared memory when warp 11 staged the row, else global memory
+          const uint4* vmv = vi != kNotStaged ? reinterpret_cast<const uint4*>(sm.vstage[sb][vi])
+                                              : reinterpret_cast<const uint4*>(v_seedmask + mrow);
           const float m2 = fmaxf(m_run, s_self);
           const float a = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m2);
           const float pself = ex2_approx(s_self - m2);
           l_run = l_run * a + pself;
 #pragma unroll
           for (int ch = 0; ch < 16; ++ch) {
-            const uint4 vv = __ldg(vmv + ch);
+            const uint4 vv = vmv[ch];
             const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
