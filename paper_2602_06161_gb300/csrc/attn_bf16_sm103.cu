@@ -15,11 +15,15 @@
 // Structure: a persistent grid of one CTA per SM; a work unit is 256 query
 // rows (two Q tiles of 128) of one head, and CTA c takes units c, c + grid,
 // c + 2 grid, ... The pipelines below run across unit boundaries, so one
-// unit's epilogue overlaps the next unit's loads and first products.
+// unit's epilogue overlaps the next unit's loads and first products. When the
+// last round of units would leave at least half of the SMs idle, its units
+// are split over two CTAs each (one Q tile per CTA, the two softmax
+// warpgroups on the two halves of the keys, merged in the epilogue).
 //   warps 0-3  softmax + epilogue of Q tile 0 (thread = row)
 //   warps 4-7  softmax + epilogue of Q tile 1
 //   warp  8    tensor-memory allocation; lane 0 issues tcgen05.mma
-//   warp  9    lane 0 issues TMA loads (Q per unit, K/V through a 2-stage ring)
+//   warp  9    lane 0 issues every TMA copy (Q per unit, K/V through a 2-stage ring,
+//              the staged output rows)
 //   warp  10   seed routing of the next unit (double-buffered slot table)
 //   warp  11   seed self scores q_i . k_i of the next unit, L2 prefetch of v_i
 // Registers: launched at 168 per thread (12 warps); the producer warpgroup
@@ -69,14 +73,34 @@ constexpr int kNotStaged = 255;
 // persistent and CTA c takes units c, c + gridDim.x, ... in order.
 struct Unit {
   int mblk, hq, b;
+  int split;   // 1: only Q tile ts of the unit, both softmax warpgroups on halves of its KV tiles
+  int ts;
 };
 
-__device__ __forceinline__ Unit unit_of(int u, int n_mblk, int Hq) {
-  Unit w;
+// Iteration it of this CTA. Units c, c + grid, ... below n_reg are whole units. When the
+// last round would leave at least half of the SMs idle, its n_split units are split instead:
+// CTA c < 2 n_split takes Q tile (c & 1) of unit n_reg + c / 2 as one more iteration, and
+// its two softmax warpgroups each take half of the KV tiles (merged in the epilogue).
+__device__ __forceinline__ bool work_of(int it, int n_reg, int n_split, int n_mblk, int Hq, Unit& w) {
+  const int c = static_cast<int>(blockIdx.x), g = static_cast<int>(gridDim.x);
+  int u = c + it * g;
+  w.split = 0;
+  w.ts = 0;
+  if (u >= n_reg) {
+    if (n_split == 0 || it * g != n_reg || c >= 2 * n_split) return false;
+    u = n_reg + (c >> 1);
+    w.split = 1;
+    w.ts = c & 1;
+  }
   w.mblk = u % n_mblk;
   w.hq = (u / n_mblk) % Hq;
   w.b = u / (n_mblk * Hq);
-  return w;
+  return true;
+}
+
+// first query row of Q tile t of a unit
+__device__ __forceinline__ int tile_row0(const Unit& w, int t) {
+  return w.mblk * kRowsPerCta + (w.split ? w.ts : t) * kBM;
 }
 
 struct AttnSmem {
@@ -105,6 +129,9 @@ struct AttnSmem {
   int slot[2][kRowsPerCta];
   Unit unit[2];                    // coordinates of the unit whose routing is in slot[sb]
   float sself[2][kRowsPerCta];     // s_self = q_i . k_i (log2-scaled) of the unit's seed rows
+  float split_m[2][kBM];           // a split unit: running max and sum per row of each KV half
+  float split_l[2][kBM];
+  uint64_t bar_split;              // ... written (all eight softmax warps)
   uint8_t vidx[2][kRowsPerCta];    // a seed row's staged value row, or kNotStaged
   alignas(16) uint8_t vstage[2][kVStageRows][kD * 2];   // masked-input value rows v_i, bf16
 };
@@ -139,7 +166,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                      const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
                      const __nv_bfloat16* __restrict__ k_seedmask,
                      const __nv_bfloat16* __restrict__ v_seedmask, const int32_t* __restrict__ seed_idx, int n_seeds,
-                     int Hq, int Hkv, int Lq_arg, int Lk, int q0_arg, int n_mblk, int n_units, float scale_log2,
+                     int Hq, int Hkv, int Lq_arg, int Lk, int q0_arg, int n_mblk, int n_reg, int n_split,
+                     float scale_log2,
                      __nv_bfloat16* __restrict__ out, float* __restrict__ lse, int* status) {
   extern __shared__ uint8_t smem_raw[];
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -176,6 +204,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sm.bar_sself_full[s], 1);
     }
     mbar_init(&sm.bar_drain, 1);
+    mbar_init(&sm.bar_split, 8);
     sm.abort = 0;
     fence_mbar_init();
     tma_prefetch_desc(&tm_q);
@@ -208,12 +237,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       // Stores unit n's output of Q tile t from the stage its last KV tile used, once the
       // tile's softmax warps have staged it; returns after the copies have read the stage.
       auto store_unit = [&](int n, int t) {
+        Unit wn;
+        work_of(n, n_reg, n_split, n_mblk, Hq, wn);
         if (!mbar_wait(&sm.bar_ostage_full[t], n & 1, &sm.abort)) return false;
-        const Unit wn = unit_of(blockIdx.x + n * gridDim.x, n_mblk, Hq);
+        // a split unit's one tile was staged by both warpgroups (one 64-column box each)
+        if (wn.split && !mbar_wait(&sm.bar_ostage_full[1], n & 1, &sm.abort)) return false;
         const int sig = (n * nkv + nkv - 1) & 1;
         const uint8_t* stage = t == 0 ? sm.k[sig] : sm.v[sig];
         for (int wq = 0; wq < 4; ++wq) {
-          const int wrow = wn.mblk * kRowsPerCta + t * kBM + wq * 32;
+          const int wrow = tile_row0(wn, t) + wq * 32;
           if (wrow < Lq) {   // rows at or past Lq fall outside the tensor and are not written
             tma_store_4d(&tm_o, stage + wq * 8192, 0, wrow, wn.hq, wn.b);
             tma_store_4d(&tm_o, stage + wq * 8192 + 4096, 64, wrow, wn.hq, wn.b);
@@ -223,8 +255,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         bulk_wait_group_read0();
         return true;
       };
-      for (int it = 0, u = blockIdx.x; u < n_units && ok; ++it, u += gridDim.x) {
-        const Unit w = unit_of(u, n_mblk, Hq);
+      const int half = nkv >> 1;
+      for (int it = 0; ok; ++it) {
+        Unit w;
+        if (!work_of(it, n_reg, n_split, n_mblk, Hq, w)) break;
         const int hkv = w.hq / group;
         // Q tile t of the unit: wait until the previous unit is done with the buffer
         auto load_q = [&](int t) {
@@ -233,12 +267,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             return false;
           mbar_arrive_expect_tx(&sm.bar_q_full[t], kTileBytes);
           for (int h = 0; h < 2; ++h)
-            tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q_full[t], 64 * h, w.mblk * kRowsPerCta + t * kBM,
-                        w.hq, w.b);
+            tma_load_4d(sm.q[t] + h * kBoxBytes, &tm_q, &sm.bar_q_full[t], 64 * h, tile_row0(w, t), w.hq, w.b);
           last_qit[t] = it;
           return true;
         };
-        for (int j = 0; j < nkv; ++j, ++G) {
+        for (int jj = 0; jj < nkv; ++jj, ++G) {
+          // KV tile of ring entry jj: in order, or for a split unit alternately from the two halves
+          const int j = !w.split ? jj : ((jj & 1) ? half + (jj >> 1) : (jj >> 1));
           const int st = G & 1, n = G >> 1;
           // tile G - 2 (same stage) was the last of a unit: the stage staged that unit's output
           const bool staged = G >= 2 && (G - 2) % nkv == nkv - 1;
@@ -254,7 +289,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int h = 0; h < 2; ++h)
             tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, j * kBN, hkv, w.b);
           last_kg = G;
-          if (j == 0 && !load_q(0)) {
+          if (jj == 0 && !load_q(0)) {
             ok = false;
             break;
           }
@@ -273,24 +308,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int h = 0; h < 2; ++h)
             tma_load_4d(sm.v[st] + h * kBoxBytes, &tm_v, &sm.bar_v_full[st], 64 * h, j * kBN, hkv, w.b);
           last_vg = G;
-          if (j == 0) {
-            for (int t = 1; t < nqt && ok; ++t) ok = load_q(t);
+          if (jj == 0) {
+            // a split unit uses its one Q tile in buffer 0 for both warpgroups
+            for (int t = 1; t < nqt && !w.split && ok; ++t) ok = load_q(t);
             if (!ok) break;
             // the next unit's Q tiles go to L2 now, so their loads at the boundary are short
-            if (u + static_cast<int>(gridDim.x) < n_units) {
-              const Unit wn = unit_of(u + gridDim.x, n_mblk, Hq);
-              for (int t = 0; t < nqt; ++t)
-                for (int h = 0; h < 2; ++h)
-                  tma_prefetch_l2_4d(&tm_q, 64 * h, wn.mblk * kRowsPerCta + t * kBM, wn.hq, wn.b);
-            }
+            Unit wn;
+            if (work_of(it + 1, n_reg, n_split, n_mblk, Hq, wn))
+              for (int t = 0; t < (wn.split ? 1 : nqt); ++t)
+                for (int h = 0; h < 2; ++h) tma_prefetch_l2_4d(&tm_q, 64 * h, tile_row0(wn, t), wn.hq, wn.b);
           }
         }
       }
-      // the units whose stages were not needed again
-      const int n_iters = (n_units - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
-                          static_cast<int>(gridDim.x);
-      for (; ok && n_stored < n_iters; ++n_stored)
-        for (int t = 0; t < nqt && ok; ++t) ok = store_unit(n_stored, t);
+      // the units whose stages were not needed again (a split unit stores its one merged tile)
+      for (; ok; ++n_stored) {
+        Unit wn;
+        if (!work_of(n_stored, n_reg, n_split, n_mblk, Hq, wn)) break;
+        for (int t = 0; t < (wn.split ? 1 : nqt) && ok; ++t) ok = store_unit(n_stored, t);
+      }
       bulk_wait_group0();
       if (!ok) {
         raise_abort(sm, status, 10);
@@ -305,19 +340,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------- seed routing ----------------
     // slot[r] of a unit = lowest seed slot naming the unit's row r, written one unit
     // ahead of the softmax warps into a double buffer.
-    for (int it = 0, u = blockIdx.x; u < n_units; ++it, u += gridDim.x) {
+    for (int it = 0;; ++it) {
+      Unit w;
+      if (!work_of(it, n_reg, n_split, n_mblk, Hq, w)) break;
       const int sb = it & 1;
       if (it >= 2 && !warp_wait(&sm.bar_slot_empty[sb], ((it >> 1) - 1) & 1, &sm.abort)) {
         if (lane == 0 && !sm.abort) raise_abort(sm, status, 40);
         break;
       }
-      const Unit w = unit_of(u, n_mblk, Hq);
       if (lane == 0) sm.unit[sb] = w;
-      route_clear(sm.slot[sb], kRowsPerCta, lane, 32);
+      // slot[t * 128 + r] belongs to query row tile_row0(w, t) + r, at memory position q0 + that
+      const int rows = w.split ? kBM : kRowsPerCta;
+      route_clear(sm.slot[sb], rows, lane, 32);
       __syncwarp();
-      // query row r of the unit sits at memory position q0 + mblk * 256 + r
-      route_scan(sm.slot[sb], seed_idx + static_cast<size_t>(w.b) * n_seeds, n_seeds,
-                 q0 + w.mblk * kRowsPerCta, kRowsPerCta, Lk, lane, 32);
+      route_scan(sm.slot[sb], seed_idx + static_cast<size_t>(w.b) * n_seeds, n_seeds, q0 + tile_row0(w, 0), rows,
+                 Lk, lane, 32);
+      if (w.split) {
+        // both warpgroups of a split unit work on the same rows
+        __syncwarp();
+        for (int r = lane; r < kBM; r += 32) sm.slot[sb][kBM + r] = sm.slot[sb][r];
+      }
       mbar_arrive(&sm.bar_slot_full[sb]);
     }
    } else if (warp == kSeedWarp) {
@@ -327,7 +369,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // row v_i copied into shared memory for the epilogue's merge (the unit's first 32 seed
     // rows; the epilogue reads any others from global memory). Runs one unit ahead of the
     // softmax warps, off their critical path.
-    for (int it = 0, u = blockIdx.x; u < n_units; ++it, u += gridDim.x) {
+    for (int it = 0;; ++it) {
+      Unit wk;
+      if (!work_of(it, n_reg, n_split, n_mblk, Hq, wk)) break;
       const int sb = it & 1;
       if (!warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort)) {
         if (lane == 0 && !sm.abort) raise_abort(sm, status, 50);
@@ -337,7 +381,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const size_t mbase = (static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds;
       int n_staged = 0;
       bool ok = true;
-      for (int t = 0; t < nqt; ++t) {
+      for (int t = 0; t < (w.split ? 1 : nqt); ++t) {
         if (!warp_wait(&sm.bar_q_full[t], it & 1, &sm.abort)) {
           ok = false;
           break;
@@ -347,7 +391,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int rc = 0; rc < kBM; rc += 32) {
           const int rr = rc + lane;
           const int sl = sm.slot[sb][t * kBM + rr];
-          const bool seed_row = sl != kNoSlot && w.mblk * kRowsPerCta + t * kBM + rr < Lq;
+          const bool seed_row = sl != kNoSlot && tile_row0(w, t) + rr < Lq;
           uint32_t pending = __ballot_sync(0xffffffffu, seed_row);
           while (pending != 0u) {
             // up to four seed rows at a time, their loads in flight together
@@ -424,9 +468,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       // unit's last products PV(0), PV(1) go first, then the new unit's S(0, 0),
       // S(1, 0), so one unit's epilogue overlaps the next unit's first products.
       // Each wait sits right after a group of products has been queued.
+      // S_t = Q(qbuf) . K(stage)^T, both K-major with 128-byte swizzle
+      auto issue_s = [&](int t, int qbuf, int kst) {
+#pragma unroll
+        for (int ks = 0; ks < kD / 16; ++ks) {
+          const uint64_t off = static_cast<uint64_t>(((ks >> 2) * kBoxBytes + (ks & 3) * 32) >> 4);
+          umma_ss(tbase + col_s(t), dq0 + qbuf * kTileDesc + off, dk0 + kst * kTileDesc + off, id_qk,
+                  ks > 0 ? 1u : 0u);
+        }
+      };
       int G = 0;
       bool ok = true;
-      for (int it = 0, u = blockIdx.x; ok; ++it, u += gridDim.x) {
+      for (int it = 0; ok; ++it) {
         if (it > 0) {
           const int pst = (G - 1) & 1;
           for (int t = 0; t < nqt; ++t) {
@@ -439,7 +492,52 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) break;
           umma_commit(&sm.bar_v_empty[pst]);
         }
-        if (u >= n_units) break;
+        Unit w;
+        if (!work_of(it, n_reg, n_split, n_mblk, Hq, w)) break;
+        if (w.split) {
+          // Split unit (always the CTA's last): tile t takes KV tiles t * half + s from ring
+          // entries G + 2 s + t, both against the Q tile in buffer 0. Every K and V tile has
+          // one user, so each product frees its own stage.
+          const int half = nkv >> 1, g0 = G;
+          for (int s = 0; s < half && ok; ++s) {
+            for (int t = 0; t < 2; ++t) {
+              const int ring = g0 + 2 * s + t;
+              if (s > 0) {
+                ok = mbar_wait(&sm.bar_p_full[t], (g0 + s - 1) & 1, &sm.abort);
+                if (!ok) break;
+                tc_fence_after_sync();
+                issue_pv(t, (ring - 2) & 1, s > 1);
+                umma_commit(&sm.bar_v_empty[(ring - 2) & 1]);
+              }
+              ok = mbar_wait(&sm.bar_k_full[ring & 1], (ring >> 1) & 1, &sm.abort);
+              if (!ok) break;
+              tc_fence_after_sync();
+              if (s == 0 && t == 0) {
+                ok = mbar_wait(&sm.bar_q_full[0], it & 1, &sm.abort);
+                if (!ok) break;
+                tc_fence_after_sync();
+              }
+              issue_s(t, 0, ring & 1);
+              umma_commit(&sm.bar_s_full[t]);
+              umma_commit(&sm.bar_k_empty[ring & 1]);
+              if (s == half - 1 && t == 1) umma_commit(&sm.bar_q_empty[0]);
+              ok = mbar_wait(&sm.bar_v_full[ring & 1], (ring >> 1) & 1, &sm.abort);
+              if (!ok) break;
+            }
+          }
+          // the last P.V products of both halves
+          for (int t = 0; t < 2 && ok; ++t) {
+            const int ring = g0 + 2 * (half - 1) + t;
+            ok = mbar_wait(&sm.bar_p_full[t], (g0 + half - 1) & 1, &sm.abort);
+            if (!ok) break;
+            tc_fence_after_sync();
+            issue_pv(t, ring & 1, half > 1);
+            umma_commit(&sm.bar_o_full[t]);
+            umma_commit(&sm.bar_v_empty[ring & 1]);
+          }
+          G = g0 + nkv;
+          break;
+        }
         for (int j = 0; j < nkv && ok; ++j, ++G) {
           const int st = G & 1, pst = (G - 1) & 1;
           for (int t = 0; t < nqt; ++t) {
@@ -460,13 +558,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (!ok) break;
               tc_fence_after_sync();
             }
-            // S_t = Q_t . K(j)^T, both K-major with 128-byte swizzle
-#pragma unroll
-            for (int ks = 0; ks < kD / 16; ++ks) {
-              const uint64_t off = static_cast<uint64_t>(((ks >> 2) * kBoxBytes + (ks & 3) * 32) >> 4);
-              umma_ss(tbase + col_s(t), dq0 + t * kTileDesc + off, dk0 + st * kTileDesc + off, id_qk,
-                      ks > 0 ? 1u : 0u);
-            }
+            issue_s(t, t, st);
             umma_commit(&sm.bar_s_full[t]);
             if (t == nqt - 1) umma_commit(&sm.bar_k_empty[st]);
             if (j == nkv - 1) umma_commit(&sm.bar_q_empty[t]);
@@ -497,30 +589,40 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       // Only what the KV loop needs stays live across it; the unit's coordinates are
       // recomputed for the epilogue.
-      for (int it = 0; blockIdx.x + it * gridDim.x < n_units && ok; ++it) {
+      for (int it = 0; ok; ++it) {
+        {
+          Unit wk;
+          if (!work_of(it, n_reg, n_split, n_mblk, Hq, wk)) break;
+        }
         const int sb = it & 1;
         int my_slot;
         int diag_j, diag_c;
+        // KV tiles of this warpgroup: all of them, or for a split unit half of them, starting
+        // at tile jbase; the tail and diagonal tiles are kept relative to jbase
+        int steps, tail_j;
         {
           ok = warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort);
           if (!ok) break;
           const Unit w = sm.unit[sb];
-          const int grow = w.mblk * kRowsPerCta + qt * kBM + r;
+          const int grow = tile_row0(w, qt) + r;
+          const int jbase = w.split ? qt * (nkv >> 1) : 0;
+          steps = w.split ? nkv >> 1 : nkv;
+          tail_j = tail_valid < kBN ? nkv - 1 - jbase : -1;   // -1: no ragged tile
           my_slot = sm.slot[sb][qt * kBM + r];
           if (grow >= Lq) my_slot = kNoSlot;
-          // the diagonal of a square launch is column r of KV tile (row0 + qt * 128) / 128; in a
-          // window a warp's 32 consecutive rows meet their diagonals in at most two KV tiles
-          diag_j = kWindow ? (q0 + grow) / kBN : (w.mblk * kRowsPerCta + qt * kBM) / kBN;
+          // the diagonal of a square launch is column r of KV tile row0 / 128 of the row's Q tile;
+          // in a window a warp's 32 consecutive rows meet their diagonals in at most two KV tiles
+          diag_j = (kWindow ? (q0 + grow) / kBN : tile_row0(w, qt) / kBN) - jbase;
           diag_c = kWindow ? (q0 + grow) % kBN : r;
         }
         const bool is_seed = my_slot != kNoSlot;
         const bool warp_seed = __any_sync(0xffffffffu, is_seed);
         const int dj_lo = kWindow ? __shfl_sync(0xffffffffu, diag_j, 0) : diag_j;
         const int dj_hi = kWindow ? __shfl_sync(0xffffffffu, diag_j, 31) : diag_j;
-        const int g0 = it * nkv;   // the CTA's KV tiles before this unit
+        const int g0 = it * nkv;   // the CTA's KV steps before this unit
         float m_run = -INFINITY, l_run = 0.0f;
 
-        for (int j = 0; j < nkv && ok; ++j) {
+        for (int j = 0; j < steps && ok; ++j) {
           ok = warp_wait(&sm.bar_s_full[qt], (g0 + j) & 1, &sm.abort);
           if (!ok) break;
           tc_fence_after_sync();
@@ -530,10 +632,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int c = 0; c < 4; ++c) tmem_ld_wait(raw[c]);
           float* s = reinterpret_cast<float*>(&raw[0][0]);
-          if (j == nkv - 1 && tail_valid < kBN) {
+          if (j == tail_j) {
+            const int valid = Lk - (nkv - 1) * kBN;
 #pragma unroll
             for (int c = 0; c < kBN; ++c)
-              if (c >= tail_valid) s[c] = -INFINITY;
+              if (c >= valid) s[c] = -INFINITY;
           }
           if (warp_seed && (j == dj_lo || j == dj_hi)) {
             // exclusion of the cached diagonal term of a seed row
@@ -612,6 +715,84 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (ok) ok = warp_wait(&sm.bar_o_full[qt], it & 1, &sm.abort);
         if (!ok) break;
+        const Unit w = sm.unit[sb];
+        if (w.split) {
+          // Split unit: the two warpgroups hold (m, l, O) of the two KV halves of the same rows.
+          // They swap (m, l) through shared memory; then each combines O = O0 2^(m0 - m) +
+          // O1 2^(m1 - m) for 64 of the 128 columns straight from tensor memory, merges a seed
+          // row's self term there, and stages its 64-column box of the rows.
+          sm.split_m[qt][r] = m_run;
+          sm.split_l[qt][r] = l_run;
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.bar_split);
+          ok = warp_wait(&sm.bar_o_full[qt ^ 1], it & 1, &sm.abort);
+          if (ok) ok = warp_wait(&sm.bar_split, 0, &sm.abort);
+          if (ok && warp_seed) ok = warp_wait(&sm.bar_sself_full[sb], (it >> 1) & 1, &sm.abort);
+          if (!ok) break;
+          tc_fence_after_sync();
+          const float m0 = sm.split_m[0][r], m1 = sm.split_m[1][r];
+          float m = fmaxf(m0, m1);
+          const float a0 = (m0 == -INFINITY) ? 0.0f : ex2_approx(m0 - m);
+          const float a1 = (m1 == -INFINITY) ? 0.0f : ex2_approx(m1 - m);
+          float l = sm.split_l[0][r] * a0 + sm.split_l[1][r] * a1;
+          const int cb = qt * 64;   // this warpgroup's columns
+          float oh[64];
+#pragma unroll
+          for (int c = 0; c < 2; ++c) {
+            uint32_t x0[32], x1[32];
+            tmem_ld32(trow + col_o(0) + cb + 32 * c, x0);
+            tmem_ld32(trow + col_o(1) + cb + 32 * c, x1);
+            tmem_ld_wait(x0);
+            tmem_ld_wait(x1);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) oh[32 * c + e] = __uint_as_float(x0[e]) * a0 + __uint_as_float(x1[e]) * a1;
+          }
+          const int grow = tile_row0(w, 0) + r;
+          if (is_seed) {
+            const float s_self = sm.sself[sb][r];
+            const int vi = sm.vidx[sb][r];
+            const size_t mrow = ((static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds + my_slot) * kD;
+            const uint4* vmv = (vi != kNotStaged ? reinterpret_cast<const uint4*>(sm.vstage[sb][vi])
+                                                 : reinterpret_cast<const uint4*>(v_seedmask + mrow)) + cb / 8;
+            const float m2 = fmaxf(m, s_self);
+            const float a = (m == -INFINITY) ? 0.0f : ex2_approx(m - m2);
+            const float pself = ex2_approx(s_self - m2);
+            l = l * a + pself;
+#pragma unroll
+            for (int ch = 0; ch < 8; ++ch) {
+              const uint4 vv = vmv[ch];
+              const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float2 vf = __bfloat1622float2(vp[e]);
+                oh[ch * 8 + 2 * e] = oh[ch * 8 + 2 * e] * a + pself * vf.x;
+                oh[ch * 8 + 2 * e + 1] = oh[ch * 8 + 2 * e + 1] * a + pself * vf.y;
+              }
+            }
+            m = m2;
+          }
+          const int sig = (g0 + nkv - 1) & 1;
+          uint8_t* stage = sm.k[sig] + (warp & 3) * (2 * 4096) + qt * 4096;
+          const float inv = 1.0f / l;
+#pragma unroll
+          for (int ch = 0; ch < 8; ++ch) {
+            uint4 v;
+            v.x = pack_bf16x2(oh[ch * 8 + 0] * inv, oh[ch * 8 + 1] * inv);
+            v.y = pack_bf16x2(oh[ch * 8 + 2] * inv, oh[ch * 8 + 3] * inv);
+            v.z = pack_bf16x2(oh[ch * 8 + 4] * inv, oh[ch * 8 + 5] * inv);
+            v.w = pack_bf16x2(oh[ch * 8 + 6] * inv, oh[ch * 8 + 7] * inv);
+            *reinterpret_cast<uint4*>(stage + lane * 128 + ((ch ^ (lane & 7)) << 4)) = v;
+          }
+          if (qt == 0 && lse != nullptr && grow < Lq)
+            lse[(static_cast<size_t>(w.b) * Hq + w.hq) * Lq + grow] = (m + log2f(l)) * 0.6931471805599453f;
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive(&sm.bar_ostage_full[qt]);
+            mbar_arrive(&sm.bar_slot_empty[sb]);
+          }
+          continue;
+        }
         // ---------------- epilogue of the unit ----------------
         // O is read into registers before this warpgroup's next P is published, so the
         // next unit's first P.V product cannot overwrite it early.
@@ -622,8 +803,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int c = 0; c < 4; ++c) tmem_ld_wait(oraw[c]);
         float* o = reinterpret_cast<float*>(&oraw[0][0]);
-        const Unit w = sm.unit[sb];
-        const int grow = w.mblk * kRowsPerCta + qt * kBM + r;
+        const int grow = tile_row0(w, qt) + r;
         if (warp_seed) {
           ok = warp_wait(&sm.bar_sself_full[sb], (it >> 1) & 1, &sm.abort);
           if (!ok) break;
@@ -704,6 +884,7 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
     return -3;
   const int n_mblk = (a.Lq + kRowsPerCta - 1) / kRowsPerCta;
   const long long n_units = static_cast<long long>(n_mblk) * a.Hq * a.B;
+  const int nkv = (a.L + kBN - 1) / kBN;
   static int n_sm = 0;
   if (n_sm == 0) {
     int dev = 0;
@@ -714,7 +895,14 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
   // unit indices advance by the grid size past the last unit: keep them inside int
   if (n_units > 0x7fffffffLL - n_sm) return -2;
   // persistent grid: one CTA per SM (1 CTA/SM fits), each looping over units
-  const long long grid = n_units < n_sm ? n_units : n_sm;
+  // The last round of units would leave at least half of the SMs idle: split its units
+  // (square launches with an even number of KV tiles), two CTAs per unit.
+  const long long rounds = n_units / n_sm, n_last = n_units % n_sm;
+  const bool window = a.Lq != a.L || a.q0 != 0;
+  const int n_split = (!window && nkv >= 2 && nkv % 2 == 0 && n_last > 0 && 2 * n_last <= n_sm)
+                          ? static_cast<int>(n_last) : 0;
+  const int n_reg = static_cast<int>(n_units) - n_split;
+  const long long grid = rounds > 0 ? n_sm : (n_split > 0 ? 2 * n_split : n_units);
   const size_t smem = sizeof(AttnSmem) + 1024;
   static bool attr_set = false;
   if (!attr_set) {
@@ -729,13 +917,12 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
     attr_set = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
-  const bool window = a.Lq != a.L || a.q0 != 0;
   auto kernel = !window       ? attn_bf16_kernel<2, false>
                 : a.Lq <= kBM ? attn_bf16_kernel<1, true>
                               : attn_bf16_kernel<2, true>;
   kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
       tq, tk, tv, to, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
-      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, static_cast<int>(n_units), scale_log2,
+      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, n_reg, n_split, scale_log2,
       static_cast<__nv_bfloat16*>(a.out), a.lse, status);
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }

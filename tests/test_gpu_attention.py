@@ -100,6 +100,7 @@ def test_f32_shapes(B, Hq, Hkv, L, D, S):
     (1, 2, 1, 129, 3),        # one key in the tail tile
     (1, 4, 2, 300, 300),      # every row a seed
     (2, 4, 4, 1000, 33),      # ragged, several CTAs
+    (1, 8, 2, 768, 20),       # GQA 4:1, every unit split over two CTAs (few units, even KV count)
 ])
 def test_bf16_shapes(B, Hq, Hkv, L, S):
     inp = W.make_attn_inputs(B, Hq, Hkv, L, 128, S, dtype="bf16", seed=B * 1000 + L + S)
@@ -128,6 +129,19 @@ def test_bf16_dominant_diagonal():
     out, lse = H.run_attn(inp)
     ref, ref_lse = H.oracle_full(inp)
     H.assert_bf16_close(out, ref, lse, ref_lse)
+
+
+def test_bf16_split_last_round():
+    """More units than SMs with a small remainder: the units of the last round are split
+    over two CTAs each (the two KV halves merged in the epilogue). Every row of the last head
+    (split units) and of the first head (whole units) against the oracle."""
+    B, Hq, Hkv, L, S = 1, 39, 39, 1024, 24
+    inp = W.make_attn_inputs(B, Hq, Hkv, L, 128, S, dtype="bf16", seed=11)
+    out, lse = H.run_attn(inp)
+    rows = list(range(L))
+    for hq in (0, Hq - 1):
+        ref, ref_lse = H.oracle_head_rows(inp, 0, hq, rows)
+        H.assert_bf16_close(out[0, hq], ref, lse[0, hq], ref_lse, f"head {hq}")
 
 
 @pytest.mark.parametrize("name", ["llada_mha_l512", "dream_gqa_l1024"])
