@@ -25,7 +25,8 @@
 //   warp  9    lane 0 issues every TMA copy (Q per unit, K/V through a 2-stage ring,
 //              the staged output rows)
 //   warp  10   seed routing of the next unit (double-buffered slot table)
-//   warp  11   seed self scores q_i . k_i of the next unit, L2 prefetch of v_i
+//   warp  11   seed self scores q_i . k_i of the next unit; copies its masked value
+//              rows v_i into shared memory for the epilogue's merge
 // Registers: launched at 168 per thread (12 warps); the producer warpgroup
 // gives back down to 136 and the two softmax warpgroups take 184 each
 // (setmaxnreg), so the 128-column softmax rows stay in registers without
