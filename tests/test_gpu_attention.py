@@ -131,6 +131,23 @@ def test_bf16_dominant_diagonal():
     H.assert_bf16_close(out, ref, lse, ref_lse)
 
 
+def test_bf16_gqa_several_rounds_and_split_sampled():
+    """GQA 5:1 with more units than SMs: every CTA runs several whole units back to back (its
+    pipelines carried across unit boundaries), then the last round's units are split over two
+    CTAs each. Seed rows and a sample of other rows of heads in the first, a middle and the
+    split last round against the oracle."""
+    B, Hq, Hkv, L, S = 2, 40, 8, 1536, 48
+    inp = W.make_attn_inputs(B, Hq, Hkv, L, 128, S, dtype="bf16", seed=21)
+    out, lse = H.run_attn(inp)
+    rng = np.random.default_rng(22)
+    for b, hq in [(0, 0), (0, 17), (1, 39)]:
+        seeds = [int(x) for x in inp.seed_idx[b] if 0 <= x < L]
+        others = rng.choice(np.setdiff1d(np.arange(L), seeds), size=48, replace=False).tolist()
+        rows = sorted(set(seeds)) + others
+        ref, ref_lse = H.oracle_head_rows(inp, b, hq, rows)
+        H.assert_bf16_close(out[b, hq, rows], ref, lse[b, hq, rows], ref_lse, f"b{b} h{hq}")
+
+
 def test_bf16_split_last_round():
     """More units than SMs with a small remainder: the units of the last round are split
     over two CTAs each (the two KV halves merged in the epilogue). Every row of the last head
