@@ -78,11 +78,31 @@ struct Unit {
   int ts;
 };
 
+// Division by a launch-invariant divisor d >= 1 through a multiply-high (the round-up method of
+// Granlund and Montgomery, "Division by invariant integers using multiplication", PLDI 1994):
+// for 0 <= u < 2^31, u / d == (umulhi(u, m) + u) >> s with s = ceil(log2 d) and
+// m = floor(2^32 (2^s - d) / d) + 1 (m < 2^32; the sum stays below 2^32). The per-unit index
+// arithmetic then runs on the integer pipes instead of the special-function unit, which the
+// softmax warps' exponentials keep busy.
+struct FastDiv {
+  uint32_t d, m, s;
+  __device__ __forceinline__ uint32_t div(uint32_t u) const { return (__umulhi(u, m) + u) >> s; }
+};
+
+// The persistent grid's unit space: n_reg whole units, n_split split ones, and the divisors
+// that decompose a unit index (n_mblk row blocks per head, Hq heads) and map a query head to
+// its KV head (Hq / Hkv query heads per KV head).
+struct UnitGrid {
+  int n_reg, n_split;
+  FastDiv mblk, hq, group;
+};
+
 // Iteration it of this CTA. Units c, c + grid, ... below n_reg are whole units. When the
 // last round would leave at least half of the SMs idle, its n_split units are split instead:
 // CTA c < 2 n_split takes Q tile (c & 1) of unit n_reg + c / 2 as one more iteration, and
 // its two softmax warpgroups each take half of the KV tiles (merged in the epilogue).
-__device__ __forceinline__ bool work_of(int it, int n_reg, int n_split, int n_mblk, int Hq, Unit& w) {
+__device__ __forceinline__ bool work_of(int it, const UnitGrid& ug, Unit& w) {
+  const int n_reg = ug.n_reg, n_split = ug.n_split;
   const int c = static_cast<int>(blockIdx.x), g = static_cast<int>(gridDim.x);
   int u = c + it * g;
   w.split = 0;
@@ -93,9 +113,11 @@ __device__ __forceinline__ bool work_of(int it, int n_reg, int n_split, int n_mb
     w.split = 1;
     w.ts = c & 1;
   }
-  w.mblk = u % n_mblk;
-  w.hq = (u / n_mblk) % Hq;
-  w.b = u / (n_mblk * Hq);
+  const uint32_t t = ug.mblk.div(static_cast<uint32_t>(u));   // (b, hq) index
+  const uint32_t b = ug.hq.div(t);
+  w.mblk = u - static_cast<int>(t * ug.mblk.d);
+  w.hq = static_cast<int>(t - b * ug.hq.d);
+  w.b = static_cast<int>(b);
   return true;
 }
 
@@ -167,7 +189,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                      const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
                      const __nv_bfloat16* __restrict__ k_seedmask,
                      const __nv_bfloat16* __restrict__ v_seedmask, const int32_t* __restrict__ seed_idx, int n_seeds,
-                     int Hq, int Hkv, int Lq_arg, int Lk, int q0_arg, int n_mblk, int n_reg, int n_split,
+                     int Hq, int Hkv, int Lq_arg, int Lk, int q0_arg, const UnitGrid ug,
                      float scale_log2,
                      __nv_bfloat16* __restrict__ out, float* __restrict__ lse, int* status) {
   extern __shared__ uint8_t smem_raw[];
@@ -175,7 +197,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
-  const int group = Hq / Hkv;
   const int nkv = (Lk + kBN - 1) / kBN;
   constexpr int nqt = NQ;
   const int Lq = kWindow ? Lq_arg : Lk;
@@ -239,7 +260,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // tile's softmax warps have staged it; returns after the copies have read the stage.
       auto store_unit = [&](int n, int t) {
         Unit wn;
-        work_of(n, n_reg, n_split, n_mblk, Hq, wn);
+        work_of(n, ug, wn);
         if (!mbar_wait(&sm.bar_ostage_full[t], n & 1, &sm.abort)) return false;
         // a split unit's one tile was staged by both warpgroups (one 64-column box each)
         if (wn.split && !mbar_wait(&sm.bar_ostage_full[1], n & 1, &sm.abort)) return false;
@@ -259,8 +280,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int half = nkv >> 1;
       for (int it = 0; ok; ++it) {
         Unit w;
-        if (!work_of(it, n_reg, n_split, n_mblk, Hq, w)) break;
-        const int hkv = w.hq / group;
+        if (!work_of(it, ug, w)) break;
+        const int hkv = static_cast<int>(ug.group.div(static_cast<uint32_t>(w.hq)));
         // Q tile t of the unit: wait until the previous unit is done with the buffer
         auto load_q = [&](int t) {
           if (it > 0 && (!mbar_wait(&sm.bar_q_empty[t], (it - 1) & 1, &sm.abort) ||
@@ -277,7 +298,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int j = !w.split ? jj : ((jj & 1) ? half + (jj >> 1) : (jj >> 1));
           const int st = G & 1, n = G >> 1;
           // tile G - 2 (same stage) was the last of a unit: the stage staged that unit's output
-          const bool staged = G >= 2 && (G - 2) % nkv == nkv - 1;
+          // (G - 2 is entry jj - 2 of this unit's ring run; every unit spans nkv entries)
+          const bool staged = G >= 2 && (nkv == 1 || jj == 1);
           if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) {
             ok = false;
             break;
@@ -315,7 +337,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
             // the next unit's Q tiles go to L2 now, so their loads at the boundary are short
             Unit wn;
-            if (work_of(it + 1, n_reg, n_split, n_mblk, Hq, wn))
+            if (work_of(it + 1, ug, wn))
               for (int t = 0; t < (wn.split ? 1 : nqt); ++t)
                 for (int h = 0; h < 2; ++h) tma_prefetch_l2_4d(&tm_q, 64 * h, tile_row0(wn, t), wn.hq, wn.b);
           }
@@ -324,7 +346,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // the units whose stages were not needed again (a split unit stores its one merged tile)
       for (; ok; ++n_stored) {
         Unit wn;
-        if (!work_of(n_stored, n_reg, n_split, n_mblk, Hq, wn)) break;
+        if (!work_of(n_stored, ug, wn)) break;
         for (int t = 0; t < (wn.split ? 1 : nqt) && ok; ++t) ok = store_unit(n_stored, t);
       }
       bulk_wait_group0();
@@ -343,7 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ahead of the softmax warps into a double buffer.
     for (int it = 0;; ++it) {
       Unit w;
-      if (!work_of(it, n_reg, n_split, n_mblk, Hq, w)) break;
+      if (!work_of(it, ug, w)) break;
       const int sb = it & 1;
       if (it >= 2 && !warp_wait(&sm.bar_slot_empty[sb], ((it >> 1) - 1) & 1, &sm.abort)) {
         if (lane == 0 && !sm.abort) raise_abort(sm, status, 40);
@@ -372,14 +394,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     // softmax warps, off their critical path.
     for (int it = 0;; ++it) {
       Unit wk;
-      if (!work_of(it, n_reg, n_split, n_mblk, Hq, wk)) break;
+      if (!work_of(it, ug, wk)) break;
       const int sb = it & 1;
       if (!warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort)) {
         if (lane == 0 && !sm.abort) raise_abort(sm, status, 50);
         break;
       }
       const Unit w = sm.unit[sb];
-      const size_t mbase = (static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds;
+      const size_t mbase = (static_cast<size_t>(w.b) * Hkv + ug.group.div(static_cast<uint32_t>(w.hq))) * n_seeds;
       int n_staged = 0;
       bool ok = true;
       for (int t = 0; t < (w.split ? 1 : nqt); ++t) {
@@ -494,7 +516,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_commit(&sm.bar_v_empty[pst]);
         }
         Unit w;
-        if (!work_of(it, n_reg, n_split, n_mblk, Hq, w)) break;
+        if (!work_of(it, ug, w)) break;
         if (w.split) {
           // Split unit (always the CTA's last): tile t takes KV tiles t * half + s from ring
           // entries G + 2 s + t, both against the Q tile in buffer 0. Every K and V tile has
@@ -593,7 +615,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; ok; ++it) {
         {
           Unit wk;
-          if (!work_of(it, n_reg, n_split, n_mblk, Hq, wk)) break;
+          if (!work_of(it, ug, wk)) break;
         }
         const int sb = it & 1;
         int my_slot;
@@ -752,7 +774,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (is_seed) {
             const float s_self = sm.sself[sb][r];
             const int vi = sm.vidx[sb][r];
-            const size_t mrow = ((static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds + my_slot) * kD;
+            const size_t mrow = ((static_cast<size_t>(w.b) * Hkv + ug.group.div(static_cast<uint32_t>(w.hq))) * n_seeds + my_slot) * kD;
             const uint4* vmv = (vi != kNotStaged ? reinterpret_cast<const uint4*>(sm.vstage[sb][vi])
                                                  : reinterpret_cast<const uint4*>(v_seedmask + mrow)) + cb / 8;
             const float m2 = fmaxf(m, s_self);
@@ -813,7 +835,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // merge the masked-input self term (k_i, v_i) of this seed row
           const float s_self = sm.sself[sb][qt * kBM + r];
           const int vi = sm.vidx[sb][qt * kBM + r];
-          const size_t mrow = ((static_cast<size_t>(w.b) * Hkv + w.hq / group) * n_seeds + my_slot) * kD;
+          const size_t mrow = ((static_cast<size_t>(w.b) * Hkv + ug.group.div(static_cast<uint32_t>(w.hq))) * n_seeds + my_slot) * kD;
           // generic loads: shared memory when warp 11 staged the row, else global memory
           const uint4* vmv = vi != kNotStaged ? reinterpret_cast<const uint4*>(sm.vstage[sb][vi])
                                               : reinterpret_cast<const uint4*>(v_seedmask + mrow);
@@ -874,6 +896,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kMmaWarp) tmem_dealloc(tbase, 512);
 }
 
+// Multiplier and shift of FastDiv for the divisor d >= 1.
+FastDiv make_fastdiv(uint32_t d) {
+  uint32_t s = 0;
+  while ((uint64_t{1} << s) < d) ++s;
+  const uint64_t m = ((uint64_t{1} << 32) * ((uint64_t{1} << s) - d)) / d + 1;
+  return FastDiv{d, static_cast<uint32_t>(m), s};
+}
+
 }  // namespace
 
 int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) {
@@ -918,12 +948,14 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
     attr_set = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
+  const UnitGrid ug{n_reg, n_split, make_fastdiv(static_cast<uint32_t>(n_mblk)),
+                    make_fastdiv(static_cast<uint32_t>(a.Hq)), make_fastdiv(static_cast<uint32_t>(a.Hq / a.Hkv))};
   auto kernel = !window       ? attn_bf16_kernel<2, false>
                 : a.Lq <= kBM ? attn_bf16_kernel<1, true>
                               : attn_bf16_kernel<2, true>;
   kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
       tq, tk, tv, to, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
-      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, n_mblk, n_reg, n_split, scale_log2,
+      a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, ug, scale_log2,
       static_cast<__nv_bfloat16*>(a.out), a.lse, status);
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
