@@ -293,9 +293,48 @@ __global__ void __launch_bounds__(kThreads, 1)
           last_qit[t] = it;
           return true;
         };
+        if (w.split) {
+          // Split unit (the CTA's last): ring entry e = 2 s + t holds KV tile t * half + s of
+          // warpgroup t's step s. Each K and V tile has one user, so K loads run a step ahead of
+          // V loads in the order the products free their stages: V(e) after P.V of step s - 1,
+          // K(e + 2) after Q.K^T of step s.
+          const int g0 = G;
+          auto load_k = [&](int e) {
+            const int g = g0 + e, st = g & 1, n = g >> 1;
+            if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) return false;
+            // entry 1 reuses the stage of the previous unit's last KV tile, which holds its output
+            if (g >= 2 && e == 1 && !store_unit(n_stored, 0)) return false;
+            mbar_arrive_expect_tx(&sm.bar_k_full[st], kTileBytes);
+            for (int h = 0; h < 2; ++h)
+              tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h,
+                          ((e & 1) * half + (e >> 1)) * kBN, hkv, w.b);
+            last_kg = g;
+            return true;
+          };
+          auto load_v = [&](int e) {
+            const int g = g0 + e, st = g & 1, n = g >> 1;
+            if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) return false;
+            if (g >= 2 && e == 1) {
+              if (nqt > 1 && !store_unit(n_stored, 1)) return false;
+              ++n_stored;
+            }
+            mbar_arrive_expect_tx(&sm.bar_v_full[st], kTileBytes);
+            for (int h = 0; h < 2; ++h)
+              tma_load_4d(sm.v[st] + h * kBoxBytes, &tm_v, &sm.bar_v_full[st], 64 * h,
+                          ((e & 1) * half + (e >> 1)) * kBN, hkv, w.b);
+            last_vg = g;
+            return true;
+          };
+          ok = load_k(0) && load_q(0) && load_k(1);
+          for (int sp = 0; sp < half && ok; ++sp) {
+            ok = load_v(2 * sp) && (sp + 1 == half || load_k(2 * sp + 2)) && load_v(2 * sp + 1) &&
+                 (sp + 1 == half || load_k(2 * sp + 3));
+          }
+          G = g0 + nkv;
+          continue;
+        }
         for (int jj = 0; jj < nkv; ++jj, ++G) {
-          // KV tile of ring entry jj: in order, or for a split unit alternately from the two halves
-          const int j = !w.split ? jj : ((jj & 1) ? half + (jj >> 1) : (jj >> 1));
+          const int j = jj;
           const int st = G & 1, n = G >> 1;
           // tile G - 2 (same stage) was the last of a unit: the stage staged that unit's output
           // (G - 2 is entry jj - 2 of this unit's ring run; every unit spans nkv entries)
@@ -520,13 +559,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (w.split) {
           // Split unit (always the CTA's last): tile t takes KV tiles t * half + s from ring
           // entries G + 2 s + t, both against the Q tile in buffer 0. Every K and V tile has
-          // one user, so each product frees its own stage.
+          // one user, so each product frees its own stage; a V tile is waited for right before
+          // its P.V product, since the TMA thread loads it only after the previous step's P.V.
           const int half = nkv >> 1, g0 = G;
           for (int s = 0; s < half && ok; ++s) {
             for (int t = 0; t < 2; ++t) {
               const int ring = g0 + 2 * s + t;
               if (s > 0) {
                 ok = mbar_wait(&sm.bar_p_full[t], (g0 + s - 1) & 1, &sm.abort);
+                if (ok) ok = mbar_wait(&sm.bar_v_full[(ring - 2) & 1], ((ring - 2) >> 1) & 1, &sm.abort);
                 if (!ok) break;
                 tc_fence_after_sync();
                 issue_pv(t, (ring - 2) & 1, s > 1);
@@ -544,14 +585,13 @@ __global__ void __launch_bounds__(kThreads, 1)
               umma_commit(&sm.bar_s_full[t]);
               umma_commit(&sm.bar_k_empty[ring & 1]);
               if (s == half - 1 && t == 1) umma_commit(&sm.bar_q_empty[0]);
-              ok = mbar_wait(&sm.bar_v_full[ring & 1], (ring >> 1) & 1, &sm.abort);
-              if (!ok) break;
             }
           }
           // the last P.V products of both halves
           for (int t = 0; t < 2 && ok; ++t) {
             const int ring = g0 + 2 * (half - 1) + t;
             ok = mbar_wait(&sm.bar_p_full[t], (g0 + half - 1) & 1, &sm.abort);
+            if (ok) ok = mbar_wait(&sm.bar_v_full[ring & 1], (ring >> 1) & 1, &sm.abort);
             if (!ok) break;
             tc_fence_after_sync();
             issue_pv(t, ring & 1, half > 1);
