@@ -333,54 +333,46 @@ __global__ void __launch_bounds__(kThreads, 1)
           G = g0 + nkv;
           continue;
         }
-        for (int jj = 0; jj < nkv; ++jj, ++G) {
-          const int j = jj;
+        // K and V tiles of ring entry jj; `staged`: the entry's stage holds the output of the unit
+        // whose last KV tile it took two entries ago, which is stored before the stage is reloaded
+        // (entry 1 of a unit, or every entry when a unit has one KV tile)
+        auto kv_entry = [&](int jj, bool staged, bool first) {
           const int st = G & 1, n = G >> 1;
-          // tile G - 2 (same stage) was the last of a unit: the stage staged that unit's output
-          // (G - 2 is entry jj - 2 of this unit's ring run; every unit spans nkv entries)
-          const bool staged = G >= 2 && (nkv == 1 || jj == 1);
-          if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) {
-            ok = false;
-            break;
-          }
-          if (staged && !store_unit(n_stored, 0)) {
-            ok = false;
-            break;
-          }
+          if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) return false;
+          if (staged && !store_unit(n_stored, 0)) return false;
           mbar_arrive_expect_tx(&sm.bar_k_full[st], kTileBytes);
           for (int h = 0; h < 2; ++h)
-            tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, j * kBN, hkv, w.b);
+            tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, jj * kBN, hkv, w.b);
           last_kg = G;
-          if (jj == 0 && !load_q(0)) {
-            ok = false;
-            break;
-          }
-          if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) {
-            ok = false;
-            break;
-          }
+          if (first && !load_q(0)) return false;
+          if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) return false;
           if (staged) {
-            if (nqt > 1 && !store_unit(n_stored, 1)) {
-              ok = false;
-              break;
-            }
+            if (nqt > 1 && !store_unit(n_stored, 1)) return false;
             ++n_stored;
           }
           mbar_arrive_expect_tx(&sm.bar_v_full[st], kTileBytes);
           for (int h = 0; h < 2; ++h)
-            tma_load_4d(sm.v[st] + h * kBoxBytes, &tm_v, &sm.bar_v_full[st], 64 * h, j * kBN, hkv, w.b);
+            tma_load_4d(sm.v[st] + h * kBoxBytes, &tm_v, &sm.bar_v_full[st], 64 * h, jj * kBN, hkv, w.b);
           last_vg = G;
-          if (jj == 0) {
-            // a split unit uses its one Q tile in buffer 0 for both warpgroups
-            for (int t = 1; t < nqt && !w.split && ok; ++t) ok = load_q(t);
-            if (!ok) break;
-            // the next unit's Q tiles go to L2 now, so their loads at the boundary are short
-            Unit wn;
-            if (work_of(it + 1, ug, wn))
-              for (int t = 0; t < (wn.split ? 1 : nqt); ++t)
-                for (int h = 0; h < 2; ++h) tma_prefetch_l2_4d(&tm_q, 64 * h, tile_row0(wn, t), wn.hq, wn.b);
-          }
+          return true;
+        };
+        ok = kv_entry(0, G >= 2 && nkv == 1, true);
+        for (int t = 1; t < nqt && ok; ++t) ok = load_q(t);
+        if (!ok) break;
+        {
+          // the next unit's Q tiles go to L2 now, so their loads at the boundary are short
+          Unit wn;
+          if (work_of(it + 1, ug, wn))
+            for (int t = 0; t < (wn.split ? 1 : nqt); ++t)
+              for (int h = 0; h < 2; ++h) tma_prefetch_l2_4d(&tm_q, 64 * h, tile_row0(wn, t), wn.hq, wn.b);
         }
+        ++G;
+        if (nkv > 1) {
+          ok = kv_entry(1, G >= 2, false);
+          ++G;
+        }
+        for (int jj = 2; jj < nkv && ok; ++jj, ++G) ok = kv_entry(jj, false, false);
+        if (!ok) break;
       }
       // the units whose stages were not needed again (a split unit stores its one merged tile)
       for (; ok; ++n_stored) {
@@ -601,23 +593,39 @@ __global__ void __launch_bounds__(kThreads, 1)
           G = g0 + nkv;
           break;
         }
-        for (int j = 0; j < nkv && ok; ++j, ++G) {
-          const int st = G & 1, pst = (G - 1) & 1;
-          for (int t = 0; t < nqt; ++t) {
-            if (j > 0) {
-              ok = mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort);
-              if (!ok) break;
-              tc_fence_after_sync();
-              issue_pv(t, pst, j > 1);
-              if (t == nqt - 1) umma_commit(&sm.bar_v_empty[pst]);
-            }
+        {
+          // step 0: the unit's Q tiles, no P.V yet
+          const int st = G & 1;
+          for (int t = 0; t < nqt && ok; ++t) {
             if (t == 0) {
               ok = mbar_wait(&sm.bar_k_full[st], (G >> 1) & 1, &sm.abort);
               if (!ok) break;
               tc_fence_after_sync();
             }
-            if (j == 0) {
-              ok = mbar_wait(&sm.bar_q_full[t], it & 1, &sm.abort);
+            ok = mbar_wait(&sm.bar_q_full[t], it & 1, &sm.abort);
+            if (!ok) break;
+            tc_fence_after_sync();
+            issue_s(t, t, st);
+            umma_commit(&sm.bar_s_full[t]);
+            if (t == nqt - 1) umma_commit(&sm.bar_k_empty[st]);
+            if (nkv == 1) umma_commit(&sm.bar_q_empty[t]);
+            if (t == 0) {
+              ok = mbar_wait(&sm.bar_v_full[st], (G >> 1) & 1, &sm.abort);
+              if (!ok) break;
+            }
+          }
+          ++G;
+        }
+        for (int j = 1; j < nkv && ok; ++j, ++G) {
+          const int st = G & 1, pst = (G - 1) & 1;
+          for (int t = 0; t < nqt; ++t) {
+            ok = mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort);
+            if (!ok) break;
+            tc_fence_after_sync();
+            issue_pv(t, pst, j > 1);
+            if (t == nqt - 1) umma_commit(&sm.bar_v_empty[pst]);
+            if (t == 0) {
+              ok = mbar_wait(&sm.bar_k_full[st], (G >> 1) & 1, &sm.abort);
               if (!ok) break;
               tc_fence_after_sync();
             }
