@@ -616,29 +616,31 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           ++G;
         }
-        for (int j = 1; j < nkv && ok; ++j, ++G) {
+        // steps 1 .. nkv - 1; the last one also releases the unit's Q tiles
+        auto kv_step = [&](int j, bool last) {
           const int st = G & 1, pst = (G - 1) & 1;
           for (int t = 0; t < nqt; ++t) {
-            ok = mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort);
-            if (!ok) break;
+            if (!mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort)) return false;
             tc_fence_after_sync();
             issue_pv(t, pst, j > 1);
             if (t == nqt - 1) umma_commit(&sm.bar_v_empty[pst]);
             if (t == 0) {
-              ok = mbar_wait(&sm.bar_k_full[st], (G >> 1) & 1, &sm.abort);
-              if (!ok) break;
+              if (!mbar_wait(&sm.bar_k_full[st], (G >> 1) & 1, &sm.abort)) return false;
               tc_fence_after_sync();
             }
             issue_s(t, t, st);
             umma_commit(&sm.bar_s_full[t]);
             if (t == nqt - 1) umma_commit(&sm.bar_k_empty[st]);
-            if (j == nkv - 1) umma_commit(&sm.bar_q_empty[t]);
-            if (t == 0) {
-              // V(j) feeds the P.V products of the next step; it was issued long before
-              ok = mbar_wait(&sm.bar_v_full[st], (G >> 1) & 1, &sm.abort);
-              if (!ok) break;
-            }
+            if (last) umma_commit(&sm.bar_q_empty[t]);
+            // V(j) feeds the P.V products of the next step; it was issued long before
+            if (t == 0 && !mbar_wait(&sm.bar_v_full[st], (G >> 1) & 1, &sm.abort)) return false;
           }
+          return true;
+        };
+        for (int j = 1; j + 1 < nkv && ok; ++j, ++G) ok = kv_step(j, false);
+        if (ok && nkv > 1) {
+          ok = kv_step(nkv - 1, true);
+          ++G;
         }
       }
       if (!ok) raise_abort(sm, status, 20);
