@@ -335,8 +335,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // K and V tiles of ring entry jj; `staged`: the entry's stage holds the output of the unit
         // whose last KV tile it took two entries ago, which is stored before the stage is reloaded
-        // (entry 1 of a unit, or every entry when a unit has one KV tile)
-        auto kv_entry = [&](int jj, bool staged, bool first) {
+        // (entry 1 of a unit). With one KV tile per unit (`store_prev`) the previous unit's output
+        // is stored instead between this entry's K and V loads: that unit can stage its output
+        // without any further load, while the next one cannot before its V tile arrives, so the
+        // staging barrier never runs two phases ahead of this thread's wait.
+        auto kv_entry = [&](int jj, bool staged, bool first, bool store_prev) {
           const int st = G & 1, n = G >> 1;
           if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) return false;
           if (staged && !store_unit(n_stored, 0)) return false;
@@ -345,6 +348,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, jj * kBN, hkv, w.b);
           last_kg = G;
           if (first && !load_q(0)) return false;
+          if (store_prev) {
+            if (!store_unit(n_stored, 0) || (nqt > 1 && !store_unit(n_stored, 1))) return false;
+            ++n_stored;
+          }
           if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) return false;
           if (staged) {
             if (nqt > 1 && !store_unit(n_stored, 1)) return false;
@@ -356,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           last_vg = G;
           return true;
         };
-        ok = kv_entry(0, G >= 2 && nkv == 1, true);
+        ok = kv_entry(0, false, true, nkv == 1 && G >= 1);
         for (int t = 1; t < nqt && ok; ++t) ok = load_q(t);
         if (!ok) break;
         {
@@ -368,10 +375,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ++G;
         if (nkv > 1) {
-          ok = kv_entry(1, G >= 2, false);
+          ok = kv_entry(1, G >= 2, false, false);
           ++G;
         }
-        for (int jj = 2; jj < nkv && ok; ++jj, ++G) ok = kv_entry(jj, false, false);
+        for (int jj = 2; jj < nkv && ok; ++jj, ++G) ok = kv_entry(jj, false, false, false);
         if (!ok) break;
       }
       // the units whose stages were not needed again (a split unit stores its one merged tile)

@@ -161,6 +161,23 @@ def test_bf16_split_last_round():
         H.assert_bf16_close(out[0, hq], ref, lse[0, hq], ref_lse, f"head {hq}")
 
 
+@pytest.mark.parametrize("B,Hq,L,heads", [
+    # one KV tile per unit, 320 units: CTAs run two or three units back to back, every ring
+    # entry reusing a stage that still holds the output of the unit two entries back
+    (8, 40, 128, [(0, 0), (3, 30), (7, 39)]),
+    # two KV tiles per unit, 160 units: one whole unit per CTA, then the last 8 units split over
+    # two CTAs each with a single KV step per warpgroup
+    (4, 40, 256, [(0, 0), (3, 31), (3, 32), (3, 39)]),
+])
+def test_bf16_short_units_several_per_cta(B, Hq, L, heads):
+    inp = W.make_attn_inputs(B, Hq, Hq, L, 128, 12, dtype="bf16", seed=B * 100 + L)
+    out, lse = H.run_attn(inp)
+    rows = list(range(L))
+    for b, hq in heads:
+        ref, ref_lse = H.oracle_head_rows(inp, b, hq, rows)
+        H.assert_bf16_close(out[b, hq], ref, lse[b, hq], ref_lse, f"L{L} b{b} h{hq}")
+
+
 @pytest.mark.parametrize("name", ["llada_mha_l512", "dream_gqa_l1024"])
 def test_bf16_named_workloads_full(name):
     inp = W.WORKLOADS[name].attn_inputs()
