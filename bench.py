@@ -382,7 +382,7 @@ def run_ours(args):
     if not args.no_secondary:
         per = {WORKLOAD: seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops)}
         kv_all = {WORKLOAD: kv_timing(api, torch, kc, vc, seeds)}
-        prefix_all = {WORKLOAD: prefix_timing(api, torch, q, kc, vc, km, vm, seeds, 64, peak)}
+        prefix_all = {WORKLOAD: prefix_timing(api, torch, q, kc, vc, km, vm, seeds, 64, peak, peaks["hbm_gbs"])}
         api.cover_attn_fwd(q, kc, vc, km, vm, seeds, out=out, lse=lse)   # the seeded pass's lse
         result["mass"] = mass_timing(api, torch, wl, q, kc, km, seeds, lse)
         del q, kc, vc, km, vm, logits
@@ -399,7 +399,8 @@ def run_ours(args):
             per[name] = seed_overhead(api, torch, oq, okc, ovc, okm, ovm, oseeds, oout, olse, ow.attn_flops)
             kv_all[name] = kv_timing(api, torch, okc, ovc, oseeds)
             if name == "dream_gqa_l1024":
-                prefix_all[name] = prefix_timing(api, torch, oq, okc, ovc, okm, ovm, oseeds, 32, peak)
+                prefix_all[name] = prefix_timing(api, torch, oq, okc, ovc, okm, ovm, oseeds, 32, peak,
+                                                 peaks["hbm_gbs"])
             del oq, okc, ovc, okm, ovm, oseeds, oout, olse
             osi = ow.score_inputs()
             if osi is not None:
@@ -560,9 +561,16 @@ def mass_timing(api, torch, wl, q, kc, km, seeds, lse, iters=20):
             "ms_total": round(sum(med.values()), 4)}
 
 
-def prefix_timing(api, torch, q, kc, vc, km, vm, seeds, Lq, peak, iters=20):
-    """Prefix-cache window (Section 6.6): the last Lq query rows (the active block) over the full memory."""
+def prefix_timing(api, torch, q, kc, vc, km, vm, seeds, Lq, peak, hbm_gbs, iters=20):
+    """Prefix-cache window (Section 6.6): the last Lq query rows (the active block) over the full memory.
+
+    A short window reads the whole memory of every head once for few query rows, so its bound is
+    HBM: the line reports GB/s of algorithmic bytes (q and out of the window, K' and V', the
+    masked seed rows, the seed list and lse) beside the tensor-core fraction.
+    """
     B, Hq, L, D = q.shape
+    Hkv = kc.shape[1]
+    S = 0 if seeds is None else seeds.shape[1]
     q0 = L - Lq
     qw = q[:, :, q0:].contiguous()
     out = torch.empty_like(qw)
@@ -581,8 +589,12 @@ def prefix_timing(api, torch, q, kc, vc, km, vm, seeds, Lq, peak, iters=20):
         ts.append(a.elapsed_time(b))
     t = statistics.median(ts)
     flops = 4.0 * B * Hq * Lq * L * D
+    nbytes = 2 * (2 * B * Hq * Lq * D) + 2 * (2 * B * Hkv * L * D) + 2 * (2 * B * Hkv * S * D) + 4 * B * S \
+        + 4 * B * Hq * Lq
+    gbs = nbytes / (t * 1e-3) / 1e9
     return {"Lq": Lq, "Lk": L, "q0": q0, "ms": round(t, 4), "tflops": round(flops / (t * 1e-3) / 1e12, 2),
-            "frac_of_peak": round(flops / (t * 1e-3) / 1e12 / peak, 4)}
+            "frac_of_peak": round(flops / (t * 1e-3) / 1e12 / peak, 4), "algorithmic_bytes": nbytes,
+            "gbs": round(gbs, 1), "frac_of_measured_hbm": round(gbs / hbm_gbs, 4)}
 
 
 def kv_timing(api, torch, k, v, seeds, iters=20):
