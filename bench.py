@@ -59,7 +59,7 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-secondary", action="store_true")
-    ap.add_argument("--only", choices=["attn", "score", "decide", "mass"], default=None,
+    ap.add_argument("--only", choices=["attn", "prefix", "score", "decide", "mass"], default=None,
                     help="time one kernel alone on the workload (for profiler captures)")
     return ap.parse_args()
 
@@ -785,6 +785,16 @@ def run_only(args):
         seeds = torch.from_numpy(ai.seed_idx).cuda()
         out, lse = torch.empty_like(q), torch.empty((wl.B, wl.Hq, wl.L), device="cuda")
         fn = lambda: api.cover_attn_fwd(q, kc, vc, km, vm, seeds, out=out, lse=lse)  # noqa: E731
+    elif args.only == "prefix":
+        # the last 64-row block over the whole memory (the bench's prefix_window line)
+        ai = wl.attn_inputs()
+        q, kc, vc = bf16_dev(ai.q, torch), bf16_dev(ai.k_cached, torch), bf16_dev(ai.v_cached, torch)
+        km, vm = bf16_dev(ai.k_seedmask, torch), bf16_dev(ai.v_seedmask, torch)
+        seeds = torch.from_numpy(ai.seed_idx).cuda()
+        q0 = wl.L - 64
+        qw = q[:, :, q0:].contiguous()
+        out, lse = torch.empty_like(qw), torch.empty((wl.B, wl.Hq, 64), device="cuda")
+        fn = lambda: api.cover_attn_fwd_prefix(qw, kc, vc, km, vm, seeds, q0=q0, out=out, lse=lse)  # noqa: E731
     elif args.only == "score":
         si = wl.score_inputs()
         logits = bf16_dev(si.logits, torch)
