@@ -44,6 +44,10 @@ def run_window(q_full, kc, vc, km, vm, seeds, q0, Lq, dtype):
     (1, 2, 2, 513, 513, 0, 8, 8),           # the whole memory: the square case
     (1, 2, 2, 400, 1, 257, 3, 1),           # a single query row that is a seed
     (1, 2, 2, 700, 300, 200, 0, 0),         # no seeds
+    # 320 one-tile units: CTAs run two or three back to back
+    (8, 40, 40, 128, 64, 64, 8, 4),         # one KV tile per unit
+    (8, 40, 8, 100, 30, 70, 6, 3),          # one ragged KV tile, GQA 5:1
+    (8, 40, 40, 256, 64, 192, 8, 4),        # two KV tiles per unit
 ])
 def test_window_bf16(B, Hq, Hkv, Lk, Lq, q0, S, inside):
     q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, S, q0, Lq, "bf16", Lk + Lq, inside)
