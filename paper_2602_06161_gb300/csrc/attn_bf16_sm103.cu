@@ -101,13 +101,19 @@ struct UnitGrid {
 // last round would leave at least half of the SMs idle, its n_split units are split instead:
 // CTA c < 2 n_split takes Q tile (c & 1) of unit n_reg + c / 2 as one more iteration, and
 // its two softmax warpgroups each take half of the KV tiles (merged in the epilogue).
+// kSplitAll (the window instance with one Q tile): when n_split > 0 every unit is split, and
+// CTA c takes units c, c + grid, ... whole, both warpgroups on the two halves of the keys.
+template <bool kSplitAll>
 __device__ __forceinline__ bool work_of(int it, const UnitGrid& ug, Unit& w) {
   const int n_reg = ug.n_reg, n_split = ug.n_split;
   const int c = static_cast<int>(blockIdx.x), g = static_cast<int>(gridDim.x);
   int u = c + it * g;
   w.split = 0;
   w.ts = 0;
-  if (u >= n_reg) {
+  if (kSplitAll && n_split > 0) {
+    if (u >= n_split) return false;
+    w.split = 1;
+  } else if (u >= n_reg) {
     if (n_split == 0 || it * g != n_reg || c >= 2 * n_split) return false;
     u = n_reg + (c >> 1);
     w.split = 1;
@@ -202,6 +208,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int Lq = kWindow ? Lq_arg : Lk;
   const int q0 = kWindow ? q0_arg : 0;
   const int tail_valid = Lk - (nkv - 1) * kBN;   // valid keys in the last KV tile (1..128)
+  // a window of at most 128 rows has one Q tile; with an even number of KV tiles its units are
+  // all split, so the second softmax warpgroup takes half of every unit's keys
+  constexpr bool kSplitAll = kWindow && NQ == 1;
+  const bool all_split = kSplitAll && ug.n_split > 0;
 
   // ---------------- prologue ----------------
   if (warp == kTmaWarp && lane == 0) {
@@ -222,7 +232,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&sm.bar_slot_full[s], 32);
-      mbar_init(&sm.bar_slot_empty[s], 4 * nqt + 1);
+      mbar_init(&sm.bar_slot_empty[s], 4 * (all_split ? 2 : nqt) + 1);
       mbar_init(&sm.bar_sself_full[s], 1);
     }
     mbar_init(&sm.bar_drain, 1);
@@ -260,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // tile's softmax warps have staged it; returns after the copies have read the stage.
       auto store_unit = [&](int n, int t) {
         Unit wn;
-        work_of(n, ug, wn);
+        work_of<kSplitAll>(n, ug, wn);
         if (!mbar_wait(&sm.bar_ostage_full[t], n & 1, &sm.abort)) return false;
         // a split unit's one tile was staged by both warpgroups (one 64-column box each)
         if (wn.split && !mbar_wait(&sm.bar_ostage_full[1], n & 1, &sm.abort)) return false;
@@ -280,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int half = nkv >> 1;
       for (int it = 0; ok; ++it) {
         Unit w;
-        if (!work_of(it, ug, w)) break;
+        if (!work_of<kSplitAll>(it, ug, w)) break;
         const int hkv = static_cast<int>(ug.group.div(static_cast<uint32_t>(w.hq)));
         // Q tile t of the unit: wait until the previous unit is done with the buffer
         auto load_q = [&](int t) {
@@ -369,7 +379,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         {
           // the next unit's Q tiles go to L2 now, so their loads at the boundary are short
           Unit wn;
-          if (work_of(it + 1, ug, wn))
+          if (work_of<kSplitAll>(it + 1, ug, wn))
             for (int t = 0; t < (wn.split ? 1 : nqt); ++t)
               for (int h = 0; h < 2; ++h) tma_prefetch_l2_4d(&tm_q, 64 * h, tile_row0(wn, t), wn.hq, wn.b);
         }
@@ -384,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // the units whose stages were not needed again (a split unit stores its one merged tile)
       for (; ok; ++n_stored) {
         Unit wn;
-        if (!work_of(n_stored, ug, wn)) break;
+        if (!work_of<kSplitAll>(n_stored, ug, wn)) break;
         for (int t = 0; t < (wn.split ? 1 : nqt) && ok; ++t) ok = store_unit(n_stored, t);
       }
       bulk_wait_group0();
@@ -403,7 +413,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ahead of the softmax warps into a double buffer.
     for (int it = 0;; ++it) {
       Unit w;
-      if (!work_of(it, ug, w)) break;
+      if (!work_of<kSplitAll>(it, ug, w)) break;
       const int sb = it & 1;
       if (it >= 2 && !warp_wait(&sm.bar_slot_empty[sb], ((it >> 1) - 1) & 1, &sm.abort)) {
         if (lane == 0 && !sm.abort) raise_abort(sm, status, 40);
@@ -432,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // softmax warps, off their critical path.
     for (int it = 0;; ++it) {
       Unit wk;
-      if (!work_of(it, ug, wk)) break;
+      if (!work_of<kSplitAll>(it, ug, wk)) break;
       const int sb = it & 1;
       if (!warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort)) {
         if (lane == 0 && !sm.abort) raise_abort(sm, status, 50);
@@ -541,7 +551,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int G = 0;
       bool ok = true;
       for (int it = 0; ok; ++it) {
-        if (it > 0) {
+        if (it > 0 && !all_split) {
           const int pst = (G - 1) & 1;
           for (int t = 0; t < nqt; ++t) {
             ok = mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort);
@@ -554,18 +564,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_commit(&sm.bar_v_empty[pst]);
         }
         Unit w;
-        if (!work_of(it, ug, w)) break;
+        if (!work_of<kSplitAll>(it, ug, w)) break;
         if (w.split) {
           // Split unit (always the CTA's last): tile t takes KV tiles t * half + s from ring
           // entries G + 2 s + t, both against the Q tile in buffer 0. Every K and V tile has
           // one user, so each product frees its own stage; a V tile is waited for right before
           // its P.V product, since the TMA thread loads it only after the previous step's P.V.
           const int half = nkv >> 1, g0 = G;
+          // P barriers complete once per warpgroup step: nkv per earlier whole unit, half per
+          // earlier split unit
+          const int pb = all_split ? it * half : g0;
           for (int s = 0; s < half && ok; ++s) {
             for (int t = 0; t < 2; ++t) {
               const int ring = g0 + 2 * s + t;
               if (s > 0) {
-                ok = mbar_wait(&sm.bar_p_full[t], (g0 + s - 1) & 1, &sm.abort);
+                ok = mbar_wait(&sm.bar_p_full[t], (pb + s - 1) & 1, &sm.abort);
                 if (ok) ok = mbar_wait(&sm.bar_v_full[(ring - 2) & 1], ((ring - 2) >> 1) & 1, &sm.abort);
                 if (!ok) break;
                 tc_fence_after_sync();
@@ -589,7 +602,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // the last P.V products of both halves
           for (int t = 0; t < 2 && ok; ++t) {
             const int ring = g0 + 2 * (half - 1) + t;
-            ok = mbar_wait(&sm.bar_p_full[t], (g0 + half - 1) & 1, &sm.abort);
+            ok = mbar_wait(&sm.bar_p_full[t], (pb + half - 1) & 1, &sm.abort);
             if (ok) ok = mbar_wait(&sm.bar_v_full[ring & 1], (ring >> 1) & 1, &sm.abort);
             if (!ok) break;
             tc_fence_after_sync();
@@ -598,6 +611,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             umma_commit(&sm.bar_v_empty[ring & 1]);
           }
           G = g0 + nkv;
+          if (all_split) continue;
           break;
         }
         {
@@ -660,8 +674,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     setmaxnreg_inc<kSoftmaxRegs>();
     // ---------------- softmax (warps 0-7) ----------------
     const int qt = warp >> 2;
-    // with a single Q tile the second tile's warps sit this launch out
-    if (qt < nqt) {
+    // with a single Q tile the second tile's warps sit this launch out, unless its units are split
+    if (qt < nqt || all_split) {
       const int r = tid & (kBM - 1);
       const uint32_t trow = tbase + (static_cast<uint32_t>((warp & 3) * 32) << 16);
       const uint32_t s_addr = trow + col_s(qt);
@@ -672,7 +686,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; ok; ++it) {
         {
           Unit wk;
-          if (!work_of(it, ug, wk)) break;
+          if (!work_of<kSplitAll>(it, ug, wk)) break;
         }
         const int sb = it & 1;
         int my_slot;
@@ -700,10 +714,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int dj_lo = kWindow ? __shfl_sync(0xffffffffu, diag_j, 0) : diag_j;
         const int dj_hi = kWindow ? __shfl_sync(0xffffffffu, diag_j, 31) : diag_j;
         const int g0 = it * nkv;   // the CTA's KV steps before this unit
+        // this warpgroup's steps before this unit (half a unit's KV tiles each when all are split)
+        const int sbase = all_split ? it * (nkv >> 1) : g0;
         float m_run = -INFINITY, l_run = 0.0f;
 
         for (int j = 0; j < steps && ok; ++j) {
-          ok = warp_wait(&sm.bar_s_full[qt], (g0 + j) & 1, &sm.abort);
+          ok = warp_wait(&sm.bar_s_full[qt], (sbase + j) & 1, &sm.abort);
           if (!ok) break;
           tc_fence_after_sync();
           uint32_t raw[4][32];
@@ -806,7 +822,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&sm.bar_split);
           ok = warp_wait(&sm.bar_o_full[qt ^ 1], it & 1, &sm.abort);
-          if (ok) ok = warp_wait(&sm.bar_split, 0, &sm.abort);
+          if (ok) ok = warp_wait(&sm.bar_split, all_split ? (it & 1) : 0, &sm.abort);
           if (ok && warp_seed) ok = warp_wait(&sm.bar_sself_full[sb], (it >> 1) & 1, &sm.abort);
           if (!ok) break;
           tc_fence_after_sync();
@@ -987,10 +1003,15 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
   // (square launches with an even number of KV tiles), two CTAs per unit.
   const long long rounds = n_units / n_sm, n_last = n_units % n_sm;
   const bool window = a.Lq != a.L || a.q0 != 0;
-  const int n_split = (!window && nkv >= 2 && nkv % 2 == 0 && n_last > 0 && 2 * n_last <= n_sm)
+  // A window of at most 128 rows has one Q tile per unit; with an even number of KV tiles every
+  // unit is split inside its CTA (both softmax warpgroups on the two halves of the keys).
+  const bool split_all = window && a.Lq <= kBM && nkv >= 2 && nkv % 2 == 0;
+  const int n_split = split_all ? static_cast<int>(n_units)
+                      : (!window && nkv >= 2 && nkv % 2 == 0 && n_last > 0 && 2 * n_last <= n_sm)
                           ? static_cast<int>(n_last) : 0;
-  const int n_reg = static_cast<int>(n_units) - n_split;
-  const long long grid = rounds > 0 ? n_sm : (n_split > 0 ? 2 * n_split : n_units);
+  const int n_reg = split_all ? 0 : static_cast<int>(n_units) - n_split;
+  const long long grid = split_all ? (rounds > 0 ? n_sm : n_units)
+                                   : (rounds > 0 ? n_sm : (n_split > 0 ? 2 * n_split : n_units));
   const size_t smem = sizeof(AttnSmem) + 1024;
   static bool attr_set = false;
   if (!attr_set) {
