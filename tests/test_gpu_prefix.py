@@ -48,6 +48,8 @@ def run_window(q_full, kc, vc, km, vm, seeds, q0, Lq, dtype):
     (8, 40, 40, 128, 64, 64, 8, 4),         # one KV tile per unit
     (8, 40, 8, 100, 30, 70, 6, 3),          # one ragged KV tile, GQA 5:1
     (8, 40, 40, 256, 64, 192, 8, 4),        # two KV tiles per unit
+    (8, 40, 40, 768, 100, 600, 8, 4),       # six KV tiles: three per warpgroup in every split unit
+    (2, 4, 2, 768, 128, 640, 10, 6),        # a full 128-row window tile, GQA 2:1
 ])
 def test_window_bf16(B, Hq, Hkv, Lk, Lq, q0, S, inside):
     q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, S, q0, Lq, "bf16", Lk + Lq, inside)
