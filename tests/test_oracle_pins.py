@@ -497,3 +497,66 @@ def test_mass_matches_the_corrected_weights():
     for j in range(n):
         assert abs(d_in[0, j] - sum(A[r, pos0 + j] for r in range(n) if masked[0, r])) < 1e-12
         assert abs(d_out[0, j] - sum(A[j, pos0 + i] for i in range(n) if drafted[0, i])) < 1e-12
+
+
+# ----------------------------------------------------------------------------
+# Row-sampled oracle (the checker of every sampled GPU parity test)
+# ----------------------------------------------------------------------------
+
+def _rows_case():
+    # two batch rows, GQA 6 query heads over 2 KV heads; batch row 1 carries a repeated and an
+    # out-of-range seed, so the per-batch routing and the lowest-slot rule are exercised
+    rng = np.random.default_rng(60)
+    q, kc, vc, km, vm, _ = rand_case(2, 6, 2, 40, 8, 5, rng=rng)
+    seeds = np.array([[3, 17, 39, 0, 22], [22, 9, 22, 41, 30]], dtype=np.int32)
+    return q, kc, vc, km, vm, seeds
+
+
+def test_rows_equal_the_full_oracle_every_head():
+    # Section 5.1 / App. B.1: each listed row of head (b, hq) is that row of the full two-view
+    # attention, for every batch row and every query head of every KV group
+    q, kc, vc, km, vm, seeds = _rows_case()
+    full, full_lse = oracle.override_attention(q, kc, vc, km, vm, seeds)
+    rows = [0, 3, 9, 17, 21, 22, 30, 39]
+    for b in range(2):
+        for hq in range(6):
+            out, lse = oracle.override_attention_rows(q, kc, vc, km, vm, seeds, b, hq, rows)
+            assert np.max(np.abs(out - full[b, hq, rows])) < 1e-13, (b, hq)
+            assert np.max(np.abs(lse - full_lse[b, hq, rows])) < 1e-13, (b, hq)
+
+
+def _rows_check_fails(rows_fn, full):
+    q, kc, vc, km, vm, seeds = _rows_case()
+    rows = [3, 9, 22, 30]
+    for b in range(2):
+        for hq in range(6):
+            out, _ = rows_fn(q, kc, vc, km, vm, seeds, b, hq, rows)
+            if np.max(np.abs(out - full[b, hq, rows])) > 1e-6:
+                return True
+    return False
+
+
+def test_planted_rows_mistakes_are_caught(monkeypatch):
+    good = orc.override_attention_rows
+    full = oracle.override_attention(*_rows_case())[0]   # computed before any mistake is planted
+    assert not _rows_check_fails(good, full)
+    # (1) a seed row keeps the cached pair on its diagonal
+    monkeypatch.setattr(orc, "view_for_row", lambda kc_h, vc_h, i, pair=None: (kc_h, vc_h))
+    assert _rows_check_fails(good, full)
+    monkeypatch.undo()
+
+    # (2) the seed routing of batch row 0 used for every batch row
+    def first_batch_seeds(q, kc, vc, km, vm, seeds, b, hq, rows):
+        s = seeds.copy()
+        s[b] = seeds[0]
+        return good(q, kc, vc, km, vm, s, b, hq, rows)
+    assert _rows_check_fails(first_batch_seeds, full)
+
+    # (3) interleaved GQA mapping (hkv = hq % Hkv) instead of contiguous groups: the query of
+    # head hq read against the KV head of head (hq % Hkv) * G under the contiguous rule
+    def interleaved(q, kc, vc, km, vm, seeds, b, hq, rows):
+        Hkv, G_ = kc.shape[1], q.shape[1] // kc.shape[1]
+        q2 = q.copy()
+        q2[b, (hq % Hkv) * G_] = q[b, hq]
+        return good(q2, kc, vc, km, vm, seeds, b, (hq % Hkv) * G_, rows)
+    assert _rows_check_fails(interleaved, full)
