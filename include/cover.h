@@ -121,6 +121,11 @@ int cover_attn_fwd_prefix_f32(const float* q, const float* k_cached, const float
 int cover_seed_route(const int32_t* seed_idx, int n_seeds, int B, int L,
                      int32_t* slot_out, uint32_t* bitmap_out, int32_t* n_invalid_out,
                      void* stream);
+/* The same function under the name the boundary's specification gives it
+ * (cover_seed_route_debug); identical arguments, results and errors. */
+int cover_seed_route_debug(const int32_t* seed_idx, int n_seeds, int B, int L,
+                           int32_t* slot_out, uint32_t* bitmap_out, int32_t* n_invalid_out,
+                           void* stream);
 
 /*
  * Bytes of device workspace cover_score_fwd needs for n_seq segments.
@@ -180,7 +185,9 @@ int cover_score_fwd(const void* logits, int N, int V, int n_seq,
  *
  * The first call on each device looks up the array's device address
  * (cudaGetSymbolAddress, with that device current); make that first call
- * before any stream capture begins. All calls share the one array: calls
+ * before any stream capture begins. The address is kept per context: after
+ * cudaDeviceReset the next call (again outside any capture) looks it up in
+ * the new context. All calls share the one array: calls
  * that overlap on the GPU (different streams, or different host threads
  * without ordering) race on it and can return wrong top-k results.
  */

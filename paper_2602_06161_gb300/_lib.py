@@ -23,6 +23,7 @@ _SIGNATURES = {
     "cover_attn_fwd_prefix": (_I, [_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
     "cover_attn_fwd_prefix_f32": (_I, [_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
     "cover_seed_route": (_I, [_P, _I, _I, _I, _P, _P, _P, _P]),
+    "cover_seed_route_debug": (_I, [_P, _I, _I, _I, _P, _P, _P, _P]),
     "cover_score_workspace_bytes": (ctypes.c_size_t, [_I]),
     "cover_score_fwd": (_I, [_P, _I, _I, _I, _P, _P, _P, _P, _I, _P, _P, _P, _P, _P, _P, _P, _P]),
     "cover_score_fwd_noalloc": (_I, [_P, _I, _I, _I, _P, _P, _P, _P, _I, _P, _P, _P, _P, _P, _P, _P]),

@@ -137,8 +137,7 @@ def cover_attn_fwd_prefix_f32(q, k_cached, v_cached, k_seedmask=None, v_seedmask
                         seed_idx, q0, out, lse, want_lse, stream)
 
 
-def cover_seed_route(seed_idx: Optional[torch.Tensor], B: int, L: int, *, device=None, stream=None):
-    """Seed routing as the kernels see it: (slot [B,L] int32, bitmap [B,ceil(L/128),4] int32 bits, n_invalid)."""
+def _seed_route(fn_name, seed_idx, B, L, device, stream):
     n_seeds = 0 if seed_idx is None else int(seed_idx.shape[1])
     if n_seeds:
         _need(seed_idx, "seed_idx", torch.int32, 2)
@@ -147,10 +146,20 @@ def cover_seed_route(seed_idx: Optional[torch.Tensor], B: int, L: int, *, device
     slot = torch.empty((B, L), dtype=torch.int32, device=device)
     bitmap = torch.empty((B, (L + 127) // 128, 4), dtype=torch.int32, device=device)
     n_invalid = torch.empty((1,), dtype=torch.int32, device=device)
-    code = _lib.load().cover_seed_route(_ptr(seed_idx) if n_seeds else None, n_seeds, B, L, _ptr(slot),
-                                        _ptr(bitmap), _ptr(n_invalid), _stream(stream))
-    _lib.check("cover_seed_route", code)
+    code = getattr(_lib.load(), fn_name)(_ptr(seed_idx) if n_seeds else None, n_seeds, B, L, _ptr(slot),
+                                         _ptr(bitmap), _ptr(n_invalid), _stream(stream))
+    _lib.check(fn_name, code)
     return slot, bitmap, n_invalid
+
+
+def cover_seed_route(seed_idx: Optional[torch.Tensor], B: int, L: int, *, device=None, stream=None):
+    """Seed routing as the kernels see it: (slot [B,L] int32, bitmap [B,ceil(L/128),4] int32 bits, n_invalid)."""
+    return _seed_route("cover_seed_route", seed_idx, B, L, device, stream)
+
+
+def cover_seed_route_debug(seed_idx: Optional[torch.Tensor], B: int, L: int, *, device=None, stream=None):
+    """cover_seed_route under its boundary-table name (same C function behind it)."""
+    return _seed_route("cover_seed_route_debug", seed_idx, B, L, device, stream)
 
 
 def cover_score_workspace_bytes(n_seq: int) -> int:

@@ -41,6 +41,7 @@
 #include <cuda_bf16.h>
 #include <math.h>
 
+#include "context.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
 #include "route.cuh"
@@ -989,13 +990,27 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
   const int n_mblk = (a.Lq + kRowsPerCta - 1) / kRowsPerCta;
   const long long n_units = static_cast<long long>(n_mblk) * a.Hq * a.B;
   const int nkv = (a.L + kBN - 1) / kBN;
-  static int n_sm = 0;
-  if (n_sm == 0) {
+  const size_t smem = sizeof(AttnSmem) + 1024;
+  // per context: the SM count, and the kernels' shared-memory limit set (a function attribute
+  // holds only in the context it was set in)
+  static ContextCache<int> setup;
+  int n_sm = 0;
+  const int rc = setup.get(&n_sm, [&](int& v) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n_sm < 1)
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v < 1)
       return -3;
-  }
+    for (auto fn : {attn_bf16_kernel<2, false>, attn_bf16_kernel<1, true>, attn_bf16_kernel<2, true>}) {
+      if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
+        return -3;
+      // the register split inside the kernel assumes exactly kLaunchRegs per thread at launch;
+      // any other count could leave setmaxnreg.inc waiting, so refuse to launch
+      cudaFuncAttributes fa;
+      if (cudaFuncGetAttributes(&fa, fn) != cudaSuccess || fa.numRegs != kLaunchRegs) return -2;
+    }
+    return 0;
+  });
+  if (rc != 0) return rc;
   // unit indices advance by the grid size past the last unit: keep them inside int
   if (n_units > 0x7fffffffLL - n_sm) return -2;
   // persistent grid: one CTA per SM (1 CTA/SM fits), each looping over units
@@ -1012,19 +1027,6 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
   const int n_reg = split_all ? 0 : static_cast<int>(n_units) - n_split;
   const long long grid = split_all ? (rounds > 0 ? n_sm : n_units)
                                    : (rounds > 0 ? n_sm : (n_split > 0 ? 2 * n_split : n_units));
-  const size_t smem = sizeof(AttnSmem) + 1024;
-  static bool attr_set = false;
-  if (!attr_set) {
-    for (auto fn : {attn_bf16_kernel<2, false>, attn_bf16_kernel<1, true>, attn_bf16_kernel<2, true>}) {
-      if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
-        return -3;
-      // the register split inside the kernel assumes exactly kLaunchRegs per thread at launch;
-      // any other count could leave setmaxnreg.inc waiting, so refuse to launch
-      cudaFuncAttributes fa;
-      if (cudaFuncGetAttributes(&fa, fn) != cudaSuccess || fa.numRegs != kLaunchRegs) return -2;
-    }
-    attr_set = true;
-  }
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
   const UnitGrid ug{n_reg, n_split, make_fastdiv(static_cast<uint32_t>(n_mblk)),
                     make_fastdiv(static_cast<uint32_t>(a.Hq)), make_fastdiv(static_cast<uint32_t>(a.Hq / a.Hkv))};

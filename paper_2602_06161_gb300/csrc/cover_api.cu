@@ -3,8 +3,7 @@
 // and dispatch to the kernel launchers.
 #include <cuda_runtime.h>
 
-#include <mutex>
-
+#include "context.cuh"
 #include "cover.h"
 #include "cover_debug.h"
 #include "kernels.cuh"
@@ -15,20 +14,20 @@ namespace {
 // [0] status code, [1] site id, [2] block id, [3] unused.
 __device__ int g_status[4];
 
-constexpr int kMaxDevices = 64;
-int* g_status_addr[kMaxDevices];
-std::mutex g_status_mu;
-
+// Device address of g_status in the current device's context: in host code the
+// symbol's name is only a host-side stand-in, so the address is looked up once
+// per context (a second device, or a context created anew after cudaDeviceReset,
+// gets its own lookup).
 int* status_block() {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
-  std::lock_guard<std::mutex> lock(g_status_mu);
-  if (g_status_addr[dev] == nullptr) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
-    g_status_addr[dev] = static_cast<int*>(p);
-  }
-  return g_status_addr[dev];
+  static cover::ContextCache<int*> cache;
+  int* p = nullptr;
+  const int rc = cache.get(&p, [](int*& v) {
+    void* a = nullptr;
+    if (cudaGetSymbolAddress(&a, g_status) != cudaSuccess || a == nullptr) return -3;
+    v = static_cast<int*>(a);
+    return 0;
+  });
+  return rc == 0 ? p : nullptr;
 }
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -124,6 +123,11 @@ int cover_seed_route(const int32_t* seed_idx, int n_seeds, int B, int L, int32_t
   if (B > 65535) return COVER_ERR_UNSUPPORTED;
   return cover::launch_seed_route(seed_idx, n_seeds, B, L, slot_out, bitmap_out, n_invalid_out,
                                   static_cast<cudaStream_t>(stream));
+}
+
+int cover_seed_route_debug(const int32_t* seed_idx, int n_seeds, int B, int L, int32_t* slot_out,
+                           uint32_t* bitmap_out, int32_t* n_invalid_out, void* stream) {
+  return cover_seed_route(seed_idx, n_seeds, B, L, slot_out, bitmap_out, n_invalid_out, stream);
 }
 
 size_t cover_score_workspace_bytes(int n_seq) { return n_seq > 0 ? sizeof(uint32_t) * static_cast<size_t>(n_seq) : 0; }

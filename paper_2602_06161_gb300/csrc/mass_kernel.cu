@@ -24,6 +24,7 @@
 #include <cuda_bf16.h>
 #include <math.h>
 
+#include "context.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
 #include "route.cuh"
@@ -331,13 +332,14 @@ int launch_attn_mass(const MassArgs& a, int* status, cudaStream_t stream) {
   float* part_in = static_cast<float*>(a.workspace);
   float* part_out = part_in + static_cast<size_t>(a.B) * a.Hq * n_qt * a.per;
   const size_t smem = sizeof(MassSmem) + 1024;
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(mass_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
-        cudaSuccess)
-      return -3;
-    attr_set = true;
-  }
+  // the shared-memory limit is a function attribute of the current context
+  static ContextCache<int> setup;
+  int unused = 0;
+  const int rc = setup.get(&unused, [&](int&) {
+    return cudaFuncSetAttribute(mass_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) ==
+                   cudaSuccess ? 0 : -3;
+  });
+  if (rc != 0) return rc;
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
   mass_kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
       tq, tk, static_cast<const __nv_bfloat16*>(a.k_seedmask), a.seed_idx, a.n_seeds, a.lse, a.Hq, a.Hkv, a.L, a.pos0,

@@ -36,8 +36,8 @@
 #include <stdint.h>
 
 #include <algorithm>
-#include <mutex>
 
+#include "context.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
 
@@ -821,13 +821,14 @@ int launch_score_impl(const ScoreArgs& a, const DecideArgs* d, int* status, cuda
   const bool aligned_rows = (a.V % 8) == 0 && (reinterpret_cast<uintptr_t>(a.logits) % 16) == 0;
   if (aligned_rows) {
     const size_t smem = std::max(keys_bytes, static_cast<size_t>(kRingStages) * kChunkBytes);
-    static bool attr = false;
-    if (!attr) {
-      if (cudaFuncSetAttribute(score_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               static_cast<int>(kRingStages * kChunkBytes)) != cudaSuccess)
-        return -3;
-      attr = true;
-    }
+    // the ring's shared-memory limit is a function attribute of the current context
+    static ContextCache<int> setup;
+    int unused = 0;
+    const int rc = setup.get(&unused, [](int&) {
+      return cudaFuncSetAttribute(score_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(kRingStages * kChunkBytes)) == cudaSuccess ? 0 : -3;
+    });
+    if (rc != 0) return rc;
     score_bulk_kernel<<<a.N, kBulkThreads, smem, stream>>>(P, status);
   } else {
     score_kernel<<<a.N, kThreads, keys_bytes, stream>>>(P);
@@ -865,23 +866,20 @@ namespace {
 // loads the library holds one copy until the process exits.
 static __device__ __align__(256) uint32_t g_noalloc_counters[kNoAllocMaxSegments];
 
-constexpr int kMaxDevicesNoAlloc = 64;
-uint32_t* g_noalloc_addr[kMaxDevicesNoAlloc];
-std::mutex g_noalloc_mu;
-
-// Device address of the counter array on the current device. In host code the
-// array's name is only a host-side stand-in, so the address is looked up once
-// per device (with that device current) and cached.
+// Device address of the counter array in the current device's context. In host
+// code the array's name is only a host-side stand-in, so the address is looked up
+// (cudaGetSymbolAddress, with the device current) the first time a context calls,
+// and again in a context created anew after cudaDeviceReset.
 uint32_t* noalloc_counters() {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevicesNoAlloc) return nullptr;
-  std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (g_noalloc_addr[dev] == nullptr) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_counters) != cudaSuccess || p == nullptr) return nullptr;
-    g_noalloc_addr[dev] = static_cast<uint32_t*>(p);
-  }
-  return g_noalloc_addr[dev];
+  static ContextCache<uint32_t*> cache;
+  uint32_t* p = nullptr;
+  const int rc = cache.get(&p, [](uint32_t*& v) {
+    void* a = nullptr;
+    if (cudaGetSymbolAddress(&a, g_noalloc_counters) != cudaSuccess || a == nullptr) return -3;
+    v = static_cast<uint32_t*>(a);
+    return 0;
+  });
+  return rc == 0 ? p : nullptr;
 }
 
 }  // namespace

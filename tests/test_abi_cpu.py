@@ -84,11 +84,21 @@ def test_score_invalid_args(lib, kw):
     assert score(lib, **kw) == -1
 
 
-def test_route_invalid_args(lib):
-    assert lib.cover_seed_route(P, 2, 0, 10, P, P, P, None) == -1
-    assert lib.cover_seed_route(P, 11, 1, 10, P, P, P, None) == -1
-    assert lib.cover_seed_route(None, 2, 1, 10, P, P, P, None) == -1
-    assert lib.cover_seed_route(P, 2, 1, 10, None, P, P, None) == -1
+@pytest.mark.parametrize("name", ["cover_seed_route", "cover_seed_route_debug"])
+def test_route_invalid_args(lib, name):
+    fn = getattr(lib, name)
+    assert fn(P, 2, 0, 10, P, P, P, None) == -1
+    assert fn(P, 11, 1, 10, P, P, P, None) == -1
+    assert fn(None, 2, 1, 10, P, P, P, None) == -1
+    assert fn(P, 2, 1, 10, None, P, P, None) == -1
+
+
+def test_boundary_names_exported(lib):
+    # the entry points the boundary's specification names, under those names
+    raw = ctypes.CDLL(build.LIB)
+    for n in ["cover_attn_fwd", "cover_attn_fwd_f32", "cover_score_fwd", "cover_seed_route_debug",
+              "cover_device_status", "cover_status_str"]:
+        assert hasattr(raw, n), n
 
 
 def test_debug_invalid_args(lib):

@@ -33,11 +33,12 @@ def test_umma_tile_operand_layouts():
                                      r2[:2, :4].tolist())
 
 
-def test_seed_routing_bit_exact():
+@pytest.mark.parametrize("route", [api.cover_seed_route, api.cover_seed_route_debug])
+def test_seed_routing_bit_exact(route):
     L = 300
     seeds = np.array([[5, 130, 5, -1, 300, 127, 128, 299],
                       [0, 0, 0, 1, 2, 3, 255, 1000]], dtype=np.int32)
-    slot, bitmap, n_inv = api.cover_seed_route(H.to_dev(seeds, "i32"), 2, L)
+    slot, bitmap, n_inv = route(H.to_dev(seeds, "i32"), 2, L)
     ref_slot, ref_bitmap, ref_inv = oracle.route_seeds(seeds, L)
     assert np.array_equal(slot.cpu().numpy(), ref_slot)
     assert np.array_equal(bitmap.cpu().numpy().view(np.uint32), ref_bitmap)

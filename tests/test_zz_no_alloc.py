@@ -70,6 +70,25 @@ def test_noalloc_matches_workspace_entry_point_twice(N, V, n_seq, k):
         _same(out, ref)
 
 
+@pytest.mark.gpu
+def test_noalloc_after_a_call_of_another_segment_shape():
+    # the shared array's counters serve whichever segments a call has: a call with many one-row
+    # segments is followed by one with a few long segments, whose top-k must still be right
+    lib = _lib.load()
+    for (N, V, n_seq, k) in [(MAX_SEQ, 64, MAX_SEQ, 1), (1024, 9000, 4, 24), (1024, 2000, 256, 3)]:
+        inp = W.make_score_inputs(N, V, n_seq, k, seed=37 + n_seq, spike_frac=0.05, with_cur_tok=True,
+                                  with_dio=True, eligible_frac=0.7)
+        logits = _dev(inp.logits, "bf16")
+        side = dict(cur_tok=_dev(inp.cur_tok, "i32"), d_in=_dev(inp.d_in, "f32"), d_out=_dev(inp.d_out, "f32"),
+                    eligible=_dev(inp.eligible, "u8"))
+        ref = api.cover_score_fwd(logits, n_seq, k, **side)
+        out = _empty_out(N, n_seq, k)
+        assert _call_noalloc(lib, logits, n_seq, k, side, out) == 0
+        torch.cuda.synchronize()
+        assert api.cover_device_status() == 0
+        _same(out, ref)
+
+
 def test_noalloc_rejects_more_sequences_than_the_array_holds():
     build.build()
     lib = ctypes.CDLL(build.LIB)
