@@ -37,6 +37,39 @@ int cover_debug_umma_tile(const void* a, const void* b, const void* p, const voi
  */
 int cover_debug_wait_timeout(int limit_us, void* stream);
 
+/*
+ * cover_attn_fwd_prefix (with Lq == Lk and q0 == 0: cover_attn_fwd) with a
+ * fault planted on purpose, to drive the bf16 attention kernel's own abort
+ * path: CTA `fault_cta` of the persistent grid leaves out the K tile load of
+ * its KV ring entry `fault_entry` (entries count the CTA's KV tiles over all
+ * of its work units, from 0), and every bounded wait of the launch gives up
+ * after `limit_us` microseconds (1 .. 2000000) instead of one second.
+ * The waits that depend on the missing tile run out: the kernel records
+ * COVER_ERR_DEVICE_TIMEOUT with the site of the first wait that gave up, every
+ * role of that CTA leaves its loop, lets the copies and tensor-core products
+ * it already issued complete, frees its tensor memory and returns; the other
+ * CTAs finish their units normally. The failed CTA's output rows are
+ * unspecified. An entry the CTA never reaches plants nothing.
+ * Arguments, layouts and errors otherwise as cover_attn_fwd_prefix (bf16).
+ */
+int cover_debug_attn_fault(const void* q, const void* k_cached, const void* v_cached,
+                           const void* k_seedmask, const void* v_seedmask,
+                           const int32_t* seed_idx, int n_seeds,
+                           int B, int Hq, int Hkv, int Lq, int Lk, int q0, int D,
+                           void* out, float* lse, int fault_cta, int fault_entry, int limit_us,
+                           void* stream);
+
+/*
+ * Like cover_device_status, and also returns where the failure came from:
+ * synchronises `stream`, copies the current device's status block to the
+ * host array detail[3] = {status code, site id, linear block id} (all 0 when
+ * nothing failed), clears it, and returns COVER_OK (COVER_ERR_CUDA if a CUDA
+ * call fails). Site ids of the bf16 attention kernel: 10 TMA thread, 20 MMA
+ * thread, 30 / 31 softmax warpgroup of Q tile 0 / 1, 40 routing warp,
+ * 50 / 51 seed-score warp.
+ */
+int cover_debug_status_detail(int32_t* detail, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

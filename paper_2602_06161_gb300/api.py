@@ -7,6 +7,7 @@ streams.
 """
 from __future__ import annotations
 
+import ctypes
 from typing import Optional
 
 import torch
@@ -89,7 +90,7 @@ def cover_attn_fwd_f32(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, 
 
 
 def _attn_prefix(fn_name, dtype, q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, q0, out, lse, want_lse,
-                 stream):
+                 stream, extra=()):
     _need(q, "q", dtype, 4)
     _need(k_cached, "k_cached", dtype, 4)
     _need(v_cached, "v_cached", dtype, 4)
@@ -118,7 +119,7 @@ def _attn_prefix(fn_name, dtype, q, k_cached, v_cached, k_seedmask, v_seedmask, 
         _ptr(q), _ptr(k_cached), _ptr(v_cached),
         _ptr(k_seedmask) if n_seeds else None, _ptr(v_seedmask) if n_seeds else None,
         _ptr(seed_idx) if n_seeds else None, n_seeds, B, Hq, Hkv, Lq, Lk, int(q0), D,
-        _ptr(out), _ptr(lse), _stream(stream))
+        _ptr(out), _ptr(lse), *extra, _stream(stream))
     _lib.check(fn_name, code)
     return out, lse
 
@@ -437,3 +438,19 @@ def cover_debug_umma_tile(a, b, p, v, *, stream=None):
 
 def cover_debug_wait_timeout(limit_us: int, *, stream=None) -> None:
     _lib.check("cover_debug_wait_timeout", _lib.load().cover_debug_wait_timeout(int(limit_us), _stream(stream)))
+
+
+def cover_debug_attn_fault(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, seed_idx=None, *, q0: int = 0,
+                           fault_cta: int, fault_entry: int, limit_us: int, out=None, lse=None, stream=None):
+    """Self-test: the bf16 attention (window form) with CTA fault_cta leaving out one K tile load and every
+    bounded wait limited to limit_us; read the outcome with cover_debug_status_detail()."""
+    return _attn_prefix("cover_debug_attn_fault", torch.bfloat16, q, k_cached, v_cached, k_seedmask, v_seedmask,
+                        seed_idx, q0, out, lse, True, stream,
+                        extra=(int(fault_cta), int(fault_entry), int(limit_us)))
+
+
+def cover_debug_status_detail(stream=None):
+    """(status code, site id, block id) of the current device's status block, which is then cleared."""
+    detail = (ctypes.c_int32 * 3)()
+    _lib.check("cover_debug_status_detail", _lib.load().cover_debug_status_detail(detail, _stream(stream)))
+    return int(detail[0]), int(detail[1]), int(detail[2])

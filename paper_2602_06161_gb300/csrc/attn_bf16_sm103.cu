@@ -79,6 +79,15 @@ struct Unit {
   int ts;
 };
 
+// Wait limit of every bounded wait of the launch, and a load the TMA thread leaves out on
+// purpose: CTA `cta` does not issue the K tile of its ring entry `entry` (its entry-th KV tile
+// over all its units). A normal launch has cta = -1 and the one-second limit; the self-test
+// entry point plants the missing load with a short limit to drive the kernel's abort path.
+struct Fault {
+  int cta, entry;
+  uint64_t wait_ns;
+};
+
 // Division by a launch-invariant divisor d >= 1 through a multiply-high (the round-up method of
 // Granlund and Montgomery, "Division by invariant integers using multiplication", PLDI 1994):
 // for 0 <= u < 2^31, u / d == (umulhi(u, m) + u) >> s with s = ceil(log2 d) and
@@ -177,8 +186,8 @@ __device__ __forceinline__ void exclude_in_chunk(float* s, uint32_t sel) {
     if ((sel >> i) & 1u) s[32 * K + i] = -INFINITY;
 }
 
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  const bool ok = mbar_wait(bar, parity, abort);
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, uint64_t limit_ns) {
+  const bool ok = mbar_wait(bar, parity, abort, limit_ns);
   return __all_sync(0xffffffffu, ok);
 }
 
@@ -190,7 +199,9 @@ __device__ __forceinline__ void raise_abort(AttnSmem& sm, int* status, int site)
 // NQ: Q tiles holding query rows (1 for a window of at most 128 rows, else 2).
 // kWindow: query row r sits at memory position q0 + r of an Lk-long memory;
 // otherwise Lq = Lk and q0 = 0 are compile-time facts.
-template <int NQ, bool kWindow>
+// kFault: the self-test instance that takes its wait limit and a planted missing load from
+// `flt`; the production instances wait up to one second and load every tile.
+template <int NQ, bool kWindow, bool kFault>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
@@ -198,7 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                      const __nv_bfloat16* __restrict__ v_seedmask, const int32_t* __restrict__ seed_idx, int n_seeds,
                      int Hq, int Hkv, int Lq_arg, int Lk, int q0_arg, const UnitGrid ug,
                      float scale_log2,
-                     __nv_bfloat16* __restrict__ out, float* __restrict__ lse, int* status) {
+                     __nv_bfloat16* __restrict__ out, float* __restrict__ lse, int* status, const Fault flt) {
   extern __shared__ uint8_t smem_raw[];
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
 
@@ -206,6 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = tid >> 5, lane = tid & 31;
   const int nkv = (Lk + kBN - 1) / kBN;
   constexpr int nqt = NQ;
+  const uint64_t wait_ns = kFault ? flt.wait_ns : kWaitLimitNs;
   const int Lq = kWindow ? Lq_arg : Lk;
   const int q0 = kWindow ? q0_arg : 0;
   const int tail_valid = Lk - (nkv - 1) * kBN;   // valid keys in the last KV tile (1..128)
@@ -266,15 +278,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       int last_kg = -1, last_vg = -1;         // last KV tiles whose K / V loads were issued
       int last_qit[kNQ] = {-1, -1};           // last units whose Q tiles were issued
       int n_stored = 0;                       // units whose output the thread has stored
+      int skipped_kg = -1;                    // the K load left out by a planted fault
+      const int fault_entry = kFault && static_cast<int>(blockIdx.x) == flt.cta ? flt.entry : -1;
       bool ok = true;
       // Stores unit n's output of Q tile t from the stage its last KV tile used, once the
       // tile's softmax warps have staged it; returns after the copies have read the stage.
       auto store_unit = [&](int n, int t) {
         Unit wn;
         work_of<kSplitAll>(n, ug, wn);
-        if (!mbar_wait(&sm.bar_ostage_full[t], n & 1, &sm.abort)) return false;
+        if (!mbar_wait(&sm.bar_ostage_full[t], n & 1, &sm.abort, wait_ns)) return false;
         // a split unit's one tile was staged by both warpgroups (one 64-column box each)
-        if (wn.split && !mbar_wait(&sm.bar_ostage_full[1], n & 1, &sm.abort)) return false;
+        if (wn.split && !mbar_wait(&sm.bar_ostage_full[1], n & 1, &sm.abort, wait_ns)) return false;
         const int sig = (n * nkv + nkv - 1) & 1;
         const uint8_t* stage = t == 0 ? sm.k[sig] : sm.v[sig];
         for (int wq = 0; wq < 4; ++wq) {
@@ -295,8 +309,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int hkv = static_cast<int>(ug.group.div(static_cast<uint32_t>(w.hq)));
         // Q tile t of the unit: wait until the previous unit is done with the buffer
         auto load_q = [&](int t) {
-          if (it > 0 && (!mbar_wait(&sm.bar_q_empty[t], (it - 1) & 1, &sm.abort) ||
-                         !mbar_wait(&sm.bar_q_read[t], (it - 1) & 1, &sm.abort)))
+          if (it > 0 && (!mbar_wait(&sm.bar_q_empty[t], (it - 1) & 1, &sm.abort, wait_ns) ||
+                         !mbar_wait(&sm.bar_q_read[t], (it - 1) & 1, &sm.abort, wait_ns)))
             return false;
           mbar_arrive_expect_tx(&sm.bar_q_full[t], kTileBytes);
           for (int h = 0; h < 2; ++h)
@@ -312,9 +326,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int g0 = G;
           auto load_k = [&](int e) {
             const int g = g0 + e, st = g & 1, n = g >> 1;
-            if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) return false;
+            if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort, wait_ns)) return false;
             // entry 1 reuses the stage of the previous unit's last KV tile, which holds its output
             if (g >= 2 && e == 1 && !store_unit(n_stored, 0)) return false;
+            if (kFault && g == fault_entry) {
+              skipped_kg = g;
+              return true;
+            }
             mbar_arrive_expect_tx(&sm.bar_k_full[st], kTileBytes);
             for (int h = 0; h < 2; ++h)
               tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h,
@@ -324,7 +342,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           };
           auto load_v = [&](int e) {
             const int g = g0 + e, st = g & 1, n = g >> 1;
-            if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) return false;
+            if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort, wait_ns)) return false;
             if (g >= 2 && e == 1) {
               if (nqt > 1 && !store_unit(n_stored, 1)) return false;
               ++n_stored;
@@ -352,18 +370,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         // staging barrier never runs two phases ahead of this thread's wait.
         auto kv_entry = [&](int jj, bool staged, bool first, bool store_prev) {
           const int st = G & 1, n = G >> 1;
-          if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort)) return false;
+          if (n >= 1 && !mbar_wait(&sm.bar_k_empty[st], (n - 1) & 1, &sm.abort, wait_ns)) return false;
           if (staged && !store_unit(n_stored, 0)) return false;
-          mbar_arrive_expect_tx(&sm.bar_k_full[st], kTileBytes);
-          for (int h = 0; h < 2; ++h)
-            tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, jj * kBN, hkv, w.b);
-          last_kg = G;
+          if (kFault && G == fault_entry) {
+            skipped_kg = G;
+          } else {
+            mbar_arrive_expect_tx(&sm.bar_k_full[st], kTileBytes);
+            for (int h = 0; h < 2; ++h)
+              tma_load_4d(sm.k[st] + h * kBoxBytes, &tm_k, &sm.bar_k_full[st], 64 * h, jj * kBN, hkv, w.b);
+            last_kg = G;
+          }
           if (first && !load_q(0)) return false;
           if (store_prev) {
             if (!store_unit(n_stored, 0) || (nqt > 1 && !store_unit(n_stored, 1))) return false;
             ++n_stored;
           }
-          if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort)) return false;
+          if (n >= 1 && !mbar_wait(&sm.bar_v_empty[st], (n - 1) & 1, &sm.abort, wait_ns)) return false;
           if (staged) {
             if (nqt > 1 && !store_unit(n_stored, 1)) return false;
             ++n_stored;
@@ -403,9 +425,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         raise_abort(sm, status, 10);
         // let every copy already issued land before the CTA's shared memory is released
         for (int t = 0; t < nqt; ++t)
-          if (last_qit[t] >= 0) mbar_wait(&sm.bar_q_full[t], last_qit[t] & 1, nullptr);
-        for (int g = max(0, last_kg - 1); g <= last_kg; ++g) mbar_wait(&sm.bar_k_full[g & 1], (g >> 1) & 1, nullptr);
-        for (int g = max(0, last_vg - 1); g <= last_vg; ++g) mbar_wait(&sm.bar_v_full[g & 1], (g >> 1) & 1, nullptr);
+          if (last_qit[t] >= 0) mbar_wait(&sm.bar_q_full[t], last_qit[t] & 1, nullptr, wait_ns);
+        for (int g = max(0, last_kg - 1); g <= last_kg; ++g)
+          if (!kFault || g != skipped_kg) mbar_wait(&sm.bar_k_full[g & 1], (g >> 1) & 1, nullptr, wait_ns);
+        for (int g = max(0, last_vg - 1); g <= last_vg; ++g)
+          mbar_wait(&sm.bar_v_full[g & 1], (g >> 1) & 1, nullptr, wait_ns);
       }
     }
    } else if (warp == kRouteWarp) {
@@ -416,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       Unit w;
       if (!work_of<kSplitAll>(it, ug, w)) break;
       const int sb = it & 1;
-      if (it >= 2 && !warp_wait(&sm.bar_slot_empty[sb], ((it >> 1) - 1) & 1, &sm.abort)) {
+      if (it >= 2 && !warp_wait(&sm.bar_slot_empty[sb], ((it >> 1) - 1) & 1, &sm.abort, wait_ns)) {
         if (lane == 0 && !sm.abort) raise_abort(sm, status, 40);
         break;
       }
@@ -445,7 +469,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       Unit wk;
       if (!work_of<kSplitAll>(it, ug, wk)) break;
       const int sb = it & 1;
-      if (!warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort)) {
+      if (!warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort, wait_ns)) {
         if (lane == 0 && !sm.abort) raise_abort(sm, status, 50);
         break;
       }
@@ -454,7 +478,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int n_staged = 0;
       bool ok = true;
       for (int t = 0; t < (w.split ? 1 : nqt); ++t) {
-        if (!warp_wait(&sm.bar_q_full[t], it & 1, &sm.abort)) {
+        if (!warp_wait(&sm.bar_q_full[t], it & 1, &sm.abort, wait_ns)) {
           ok = false;
           break;
         }
@@ -555,7 +579,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (it > 0 && !all_split) {
           const int pst = (G - 1) & 1;
           for (int t = 0; t < nqt; ++t) {
-            ok = mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort);
+            ok = mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort, wait_ns);
             if (!ok) break;
             tc_fence_after_sync();
             issue_pv(t, pst, nkv > 1);
@@ -579,18 +603,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int t = 0; t < 2; ++t) {
               const int ring = g0 + 2 * s + t;
               if (s > 0) {
-                ok = mbar_wait(&sm.bar_p_full[t], (pb + s - 1) & 1, &sm.abort);
-                if (ok) ok = mbar_wait(&sm.bar_v_full[(ring - 2) & 1], ((ring - 2) >> 1) & 1, &sm.abort);
+                ok = mbar_wait(&sm.bar_p_full[t], (pb + s - 1) & 1, &sm.abort, wait_ns);
+                if (ok) ok = mbar_wait(&sm.bar_v_full[(ring - 2) & 1], ((ring - 2) >> 1) & 1, &sm.abort, wait_ns);
                 if (!ok) break;
                 tc_fence_after_sync();
                 issue_pv(t, (ring - 2) & 1, s > 1);
                 umma_commit(&sm.bar_v_empty[(ring - 2) & 1]);
               }
-              ok = mbar_wait(&sm.bar_k_full[ring & 1], (ring >> 1) & 1, &sm.abort);
+              ok = mbar_wait(&sm.bar_k_full[ring & 1], (ring >> 1) & 1, &sm.abort, wait_ns);
               if (!ok) break;
               tc_fence_after_sync();
               if (s == 0 && t == 0) {
-                ok = mbar_wait(&sm.bar_q_full[0], it & 1, &sm.abort);
+                ok = mbar_wait(&sm.bar_q_full[0], it & 1, &sm.abort, wait_ns);
                 if (!ok) break;
                 tc_fence_after_sync();
               }
@@ -603,8 +627,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           // the last P.V products of both halves
           for (int t = 0; t < 2 && ok; ++t) {
             const int ring = g0 + 2 * (half - 1) + t;
-            ok = mbar_wait(&sm.bar_p_full[t], (pb + half - 1) & 1, &sm.abort);
-            if (ok) ok = mbar_wait(&sm.bar_v_full[ring & 1], (ring >> 1) & 1, &sm.abort);
+            ok = mbar_wait(&sm.bar_p_full[t], (pb + half - 1) & 1, &sm.abort, wait_ns);
+            if (ok) ok = mbar_wait(&sm.bar_v_full[ring & 1], (ring >> 1) & 1, &sm.abort, wait_ns);
             if (!ok) break;
             tc_fence_after_sync();
             issue_pv(t, ring & 1, half > 1);
@@ -620,11 +644,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int st = G & 1;
           for (int t = 0; t < nqt && ok; ++t) {
             if (t == 0) {
-              ok = mbar_wait(&sm.bar_k_full[st], (G >> 1) & 1, &sm.abort);
+              ok = mbar_wait(&sm.bar_k_full[st], (G >> 1) & 1, &sm.abort, wait_ns);
               if (!ok) break;
               tc_fence_after_sync();
             }
-            ok = mbar_wait(&sm.bar_q_full[t], it & 1, &sm.abort);
+            ok = mbar_wait(&sm.bar_q_full[t], it & 1, &sm.abort, wait_ns);
             if (!ok) break;
             tc_fence_after_sync();
             issue_s(t, t, st);
@@ -632,7 +656,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (t == nqt - 1) umma_commit(&sm.bar_k_empty[st]);
             if (nkv == 1) umma_commit(&sm.bar_q_empty[t]);
             if (t == 0) {
-              ok = mbar_wait(&sm.bar_v_full[st], (G >> 1) & 1, &sm.abort);
+              ok = mbar_wait(&sm.bar_v_full[st], (G >> 1) & 1, &sm.abort, wait_ns);
               if (!ok) break;
             }
           }
@@ -642,12 +666,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         auto kv_step = [&](int j, bool last) {
           const int st = G & 1, pst = (G - 1) & 1;
           for (int t = 0; t < nqt; ++t) {
-            if (!mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort)) return false;
+            if (!mbar_wait(&sm.bar_p_full[t], (G - 1) & 1, &sm.abort, wait_ns)) return false;
             tc_fence_after_sync();
             issue_pv(t, pst, j > 1);
             if (t == nqt - 1) umma_commit(&sm.bar_v_empty[pst]);
             if (t == 0) {
-              if (!mbar_wait(&sm.bar_k_full[st], (G >> 1) & 1, &sm.abort)) return false;
+              if (!mbar_wait(&sm.bar_k_full[st], (G >> 1) & 1, &sm.abort, wait_ns)) return false;
               tc_fence_after_sync();
             }
             issue_s(t, t, st);
@@ -655,7 +679,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (t == nqt - 1) umma_commit(&sm.bar_k_empty[st]);
             if (last) umma_commit(&sm.bar_q_empty[t]);
             // V(j) feeds the P.V products of the next step; it was issued long before
-            if (t == 0 && !mbar_wait(&sm.bar_v_full[st], (G >> 1) & 1, &sm.abort)) return false;
+            if (t == 0 && !mbar_wait(&sm.bar_v_full[st], (G >> 1) & 1, &sm.abort, wait_ns)) return false;
           }
           return true;
         };
@@ -668,7 +692,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) raise_abort(sm, status, 20);
       // all tensor-core work of this CTA must finish before tensor memory is released
       umma_commit(&sm.bar_drain);
-      mbar_wait(&sm.bar_drain, 0, nullptr);
+      mbar_wait(&sm.bar_drain, 0, nullptr, wait_ns);
     }
    }
   } else {
@@ -696,7 +720,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // at tile jbase; the tail and diagonal tiles are kept relative to jbase
         int steps, tail_j;
         {
-          ok = warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort);
+          ok = warp_wait(&sm.bar_slot_full[sb], (it >> 1) & 1, &sm.abort, wait_ns);
           if (!ok) break;
           const Unit w = sm.unit[sb];
           const int grow = tile_row0(w, qt) + r;
@@ -720,7 +744,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         float m_run = -INFINITY, l_run = 0.0f;
 
         for (int j = 0; j < steps && ok; ++j) {
-          ok = warp_wait(&sm.bar_s_full[qt], (sbase + j) & 1, &sm.abort);
+          ok = warp_wait(&sm.bar_s_full[qt], (sbase + j) & 1, &sm.abort, wait_ns);
           if (!ok) break;
           tc_fence_after_sync();
           uint32_t raw[4][32];
@@ -810,7 +834,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_before_sync();
           mbar_arrive(&sm.bar_p_full[qt]);
         }
-        if (ok) ok = warp_wait(&sm.bar_o_full[qt], it & 1, &sm.abort);
+        if (ok) ok = warp_wait(&sm.bar_o_full[qt], it & 1, &sm.abort, wait_ns);
         if (!ok) break;
         const Unit w = sm.unit[sb];
         if (w.split) {
@@ -822,9 +846,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           sm.split_l[qt][r] = l_run;
           __syncwarp();
           if (lane == 0) mbar_arrive(&sm.bar_split);
-          ok = warp_wait(&sm.bar_o_full[qt ^ 1], it & 1, &sm.abort);
-          if (ok) ok = warp_wait(&sm.bar_split, all_split ? (it & 1) : 0, &sm.abort);
-          if (ok && warp_seed) ok = warp_wait(&sm.bar_sself_full[sb], (it >> 1) & 1, &sm.abort);
+          ok = warp_wait(&sm.bar_o_full[qt ^ 1], it & 1, &sm.abort, wait_ns);
+          if (ok) ok = warp_wait(&sm.bar_split, all_split ? (it & 1) : 0, &sm.abort, wait_ns);
+          if (ok && warp_seed) ok = warp_wait(&sm.bar_sself_full[sb], (it >> 1) & 1, &sm.abort, wait_ns);
           if (!ok) break;
           tc_fence_after_sync();
           const float m0 = sm.split_m[0][r], m1 = sm.split_m[1][r];
@@ -902,7 +926,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         float* o = reinterpret_cast<float*>(&oraw[0][0]);
         const int grow = tile_row0(w, qt) + r;
         if (warp_seed) {
-          ok = warp_wait(&sm.bar_sself_full[sb], (it >> 1) & 1, &sm.abort);
+          ok = warp_wait(&sm.bar_sself_full[sb], (it >> 1) & 1, &sm.abort, wait_ns);
           if (!ok) break;
         }
         if (is_seed) {
@@ -1000,7 +1024,9 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v < 1)
       return -3;
-    for (auto fn : {attn_bf16_kernel<2, false>, attn_bf16_kernel<1, true>, attn_bf16_kernel<2, true>}) {
+    for (auto fn : {attn_bf16_kernel<2, false, false>, attn_bf16_kernel<1, true, false>,
+                    attn_bf16_kernel<2, true, false>, attn_bf16_kernel<2, false, true>,
+                    attn_bf16_kernel<1, true, true>, attn_bf16_kernel<2, true, true>}) {
       if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
         return -3;
       // the register split inside the kernel assumes exactly kLaunchRegs per thread at launch;
@@ -1030,13 +1056,15 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream) 
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
   const UnitGrid ug{n_reg, n_split, make_fastdiv(static_cast<uint32_t>(n_mblk)),
                     make_fastdiv(static_cast<uint32_t>(a.Hq)), make_fastdiv(static_cast<uint32_t>(a.Hq / a.Hkv))};
-  auto kernel = !window       ? attn_bf16_kernel<2, false>
-                : a.Lq <= kBM ? attn_bf16_kernel<1, true>
-                              : attn_bf16_kernel<2, true>;
+  const bool fault = a.fault_cta >= 0 || a.wait_ns > 0;
+  auto kernel = !window       ? (fault ? attn_bf16_kernel<2, false, true> : attn_bf16_kernel<2, false, false>)
+                : a.Lq <= kBM ? (fault ? attn_bf16_kernel<1, true, true> : attn_bf16_kernel<1, true, false>)
+                              : (fault ? attn_bf16_kernel<2, true, true> : attn_bf16_kernel<2, true, false>);
   kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(
       tq, tk, tv, to, static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask),
       a.seed_idx, a.n_seeds, a.Hq, a.Hkv, a.Lq, a.L, a.q0, ug, scale_log2,
-      static_cast<__nv_bfloat16*>(a.out), a.lse, status);
+      static_cast<__nv_bfloat16*>(a.out), a.lse, status,
+      Fault{a.fault_cta, a.fault_entry, a.wait_ns > 0 ? a.wait_ns : kWaitLimitNs});
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
 

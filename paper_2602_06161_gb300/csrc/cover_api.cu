@@ -296,16 +296,31 @@ int cover_attn_mass_fwd(const void* q, const void* k_cached, const void* k_seedm
   return rc == -2 ? COVER_ERR_UNSUPPORTED : rc == 0 ? COVER_OK : COVER_ERR_CUDA;
 }
 
-int cover_device_status(void* stream) {
+// Synchronises the stream, reads the status block into host[4] and clears it.
+static int read_status(void* stream, int* host) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int* st = status_block();
   if (st == nullptr) return COVER_ERR_CUDA;
   if (cudaStreamSynchronize(s) != cudaSuccess) return COVER_ERR_CUDA;
-  int host[4] = {0, 0, 0, 0};
-  if (cudaMemcpyAsync(host, st, sizeof(host), cudaMemcpyDeviceToHost, s) != cudaSuccess) return COVER_ERR_CUDA;
-  if (cudaMemsetAsync(st, 0, sizeof(host), s) != cudaSuccess) return COVER_ERR_CUDA;
+  if (cudaMemcpyAsync(host, st, 4 * sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess) return COVER_ERR_CUDA;
+  if (cudaMemsetAsync(st, 0, 4 * sizeof(int), s) != cudaSuccess) return COVER_ERR_CUDA;
   if (cudaStreamSynchronize(s) != cudaSuccess) return COVER_ERR_CUDA;
-  return host[0];
+  return COVER_OK;
+}
+
+int cover_device_status(void* stream) {
+  int host[4] = {0, 0, 0, 0};
+  const int rc = read_status(stream, host);
+  return rc != COVER_OK ? rc : host[0];
+}
+
+int cover_debug_status_detail(int32_t* detail, void* stream) {
+  if (detail == nullptr) return COVER_ERR_INVALID_ARG;
+  int host[4] = {0, 0, 0, 0};
+  const int rc = read_status(stream, host);
+  if (rc != COVER_OK) return rc;
+  for (int i = 0; i < 3; ++i) detail[i] = host[i];
+  return COVER_OK;
 }
 
 const char* cover_status_str(int code) {
@@ -329,6 +344,27 @@ int cover_debug_umma_tile(const void* a, const void* b, const void* p, const voi
   int* st = status_block();
   if (st == nullptr) return COVER_ERR_CUDA;
   return cover::launch_umma_tile(a, b, p, v, c1, c2, st, static_cast<cudaStream_t>(stream));
+}
+
+int cover_debug_attn_fault(const void* q, const void* k_cached, const void* v_cached, const void* k_seedmask,
+                           const void* v_seedmask, const int32_t* seed_idx, int n_seeds, int B, int Hq, int Hkv,
+                           int Lq, int Lk, int q0, int D, void* out, float* lse, int fault_cta, int fault_entry,
+                           int limit_us, void* stream) {
+  if (limit_us < 1 || limit_us > 2000000) return COVER_ERR_INVALID_ARG;
+  int rc = check_window(Lq, Lk, q0);
+  if (rc != COVER_OK) return rc;
+  rc = check_attn_args(q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
+                       16);
+  if (rc != COVER_OK) return rc;
+  if (D != 128) return COVER_ERR_UNSUPPORTED;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
+                    Lq, q0};
+  a.fault_cta = fault_cta;
+  a.fault_entry = fault_entry;
+  a.wait_ns = static_cast<uint64_t>(limit_us) * 1000ull;
+  return cover::launch_attn_bf16_sm103(a, st, static_cast<cudaStream_t>(stream));
 }
 
 int cover_debug_wait_timeout(int limit_us, void* stream) {

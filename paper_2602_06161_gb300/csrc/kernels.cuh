@@ -21,6 +21,11 @@ struct AttnArgs {
   float* lse;
   int Lq = 0;             // query rows; query row r sits at memory position q0 + r
   int q0 = 0;
+  // self-test only (bf16 kernel): CTA fault_cta leaves out the K load of its KV ring entry
+  // fault_entry, and every bounded wait gives up after wait_ns (0: the default limit)
+  int fault_cta = -1;
+  int fault_entry = -1;
+  uint64_t wait_ns = 0;
 };
 
 int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream);

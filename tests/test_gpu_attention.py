@@ -11,6 +11,7 @@ import oracle
 from paper_2602_06161_gb300 import api
 from paper_2602_06161_gb300 import workloads as W
 from tests import _gpu as H
+from tests import _oracle_pool as OP
 
 pytestmark = pytest.mark.gpu
 
@@ -201,6 +202,28 @@ def test_bf16_named_workloads_sampled(name):
         rows = seeds + others
         ref, ref_lse = H.oracle_head_rows(inp, b, hq, rows)
         H.assert_bf16_close(out[b, hq, rows], ref, lse[b, hq, rows], ref_lse, f"{name} b{b} h{hq}")
+
+
+@pytest.mark.parametrize("name", ["llada_b8_l2048", "gqa_l8192_stress"])
+def test_bf16_named_workloads_whole_tensor(name):
+    """Full-size launch compared with the oracle on every element of out and lse (every head,
+    every row; the oracle's heads run in spawned worker processes)."""
+    inp = W.WORKLOADS[name].attn_inputs()
+    args = _dev_inputs(inp)
+    out, lse = api.cover_attn_fwd(*args)
+    torch.cuda.synchronize()
+    assert api.cover_device_status() == 0
+    out_bits = out.view(torch.int16).cpu().numpy().view(np.uint16)
+    lse_h = lse.cpu().numpy()
+    del out, lse, args
+    G = inp.Hq // inp.Hkv
+    heads = [(b, hq) for b in range(inp.B) for hq in range(inp.Hq)]
+    tasks = ((inp.q[b, hq], inp.k_cached[b, hq // G], inp.v_cached[b, hq // G], inp.k_seedmask[b, hq // G],
+              inp.v_seedmask[b, hq // G], inp.seed_idx[b], out_bits[b, hq], lse_h[b, hq]) for b, hq in heads)
+    dmax, dmean, lmax, n = OP.check_heads(tasks, len(heads))
+    print(f"{name}: {n} heads, max |d| {dmax:.3e}, mean |d| {dmean:.3e}, lse max |d| {lmax:.3e}")
+    assert n == len(heads)
+    assert dmax <= H.TOL_BF16_MAX and dmean <= H.TOL_BF16_MEAN and lmax <= H.TOL_LSE, (dmax, dmean, lmax)
 
 
 # ----------------------------------------------------------------------------
