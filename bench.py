@@ -632,38 +632,49 @@ def kv_timing(api, torch, k, v, seeds, iters=20):
             "gbs_override": round(2 * g_bytes / (t_o * 1e-3) / 1e9, 1)}
 
 
-def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, iters=20):
-    """Median attention time with the configured seeds vs. the same tensors with no seeds."""
+def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, pairs=200):
+    """Attention time with the configured seeds vs. the same tensors with no seeds.
+
+    `pairs` seeded / unseeded launches are interleaved (the order alternating from pair to pair),
+    each timed alone with CUDA events behind a device-side spin, so slow drifts of clock or
+    temperature hit both arms alike. The overhead is the median of the per-pair ratios, with
+    their 10th / 90th percentiles as its spread; the minimum and the median of each arm and the
+    ratio of the minima are reported beside it (on launches of ~15 us a single fast outlier
+    moves the minima by several percent, the pair median does not move).
+    """
     stream = torch.cuda.current_stream()
 
-    def timed(with_seeds):
-        for _ in range(3):
-            if with_seeds:
-                api.cover_attn_fwd(q, kc, vc, km, vm, seeds, out=out, lse=lse)
-            else:
-                api.cover_attn_fwd(q, kc, vc, out=out, lse=lse)
-        ts = []
-        for _ in range(iters):
+    def launch(with_seeds):
+        if with_seeds:
+            api.cover_attn_fwd(q, kc, vc, km, vm, seeds, out=out, lse=lse)
+        else:
+            api.cover_attn_fwd(q, kc, vc, out=out, lse=lse)
+
+    for _ in range(3):
+        launch(True)
+        launch(False)
+    ts = {True: [], False: []}
+    for i in range(pairs):
+        for with_seeds in ((True, False) if i % 2 == 0 else (False, True)):
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             busy_ahead(torch)
             a.record(stream)
-            if with_seeds:
-                api.cover_attn_fwd(q, kc, vc, km, vm, seeds, out=out, lse=lse)
-            else:
-                api.cover_attn_fwd(q, kc, vc, out=out, lse=lse)
+            launch(with_seeds)
             b.record(stream)
             torch.cuda.synchronize()
-            ts.append(a.elapsed_time(b))
-        return statistics.median(ts)
-
-    t_seed = timed(True)
-    t_none = timed(False)
-    t_seed = min(t_seed, timed(True))   # alternate once more to cancel drift
-    t_none = min(t_none, timed(False))
+            ts[with_seeds].append(a.elapsed_time(b))
+    ratios = sorted(s / n - 1.0 for s, n in zip(ts[True], ts[False]))
+    t_seed, t_none = min(ts[True]), min(ts[False])
+    pct = lambda p: ratios[min(len(ratios) - 1, int(p * len(ratios)))]  # noqa: E731
     return {"ms_seeded": round(t_seed, 4), "ms_no_seed": round(t_none, 4),
+            "ms_seeded_median": round(statistics.median(ts[True]), 4),
+            "ms_no_seed_median": round(statistics.median(ts[False]), 4),
             "tflops_seeded": round(flops / (t_seed * 1e-3) / 1e12, 2),
             "tflops_no_seed": round(flops / (t_none * 1e-3) / 1e12, 2),
-            "overhead": round((t_seed - t_none) / t_none, 4)}
+            "overhead": round(statistics.median(ratios), 4),
+            "overhead_p10_p90": [round(pct(0.1), 4), round(pct(0.9), 4)],
+            "overhead_of_minima": round((t_seed - t_none) / t_none, 4),
+            "pairs": pairs}
 
 
 # ----------------------------------------------------------------------------
