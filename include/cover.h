@@ -318,8 +318,9 @@ int cover_score_decide_fwd(const void* logits, int N, int V, int n_seq,
  * diagonal uses its masked-input key (the leave-one-out view; lse is the one
  * cover_attn_fwd wrote, that of the corrected distribution). Only response
  * queries and response keys contribute. Tensor-core recomputation of the
- * per x per block of every head; partial sums per head are added in a fixed
- * order, so the result is deterministic.
+ * per x per block of every head (once per orientation, so that both sums are
+ * row sums); partial sums per head are added in a fixed order, so the result
+ * is deterministic.
  * q [B, Hq, L, 128], k_cached [B, Hkv, L, 128], k_seedmask [B, Hkv, n_seeds,
  * 128] bf16; seed_idx int32 [B, n_seeds]; lse float [B, Hq, L]; tok int32,
  * flags uint8 [B * per] (cover_score_decide_fwd's state after the update
@@ -328,8 +329,10 @@ int cover_score_decide_fwd(const void* logits, int N, int V, int n_seq,
  * initialisation needed. All device pointers, owned by the caller.
  * Errors: COVER_ERR_INVALID_ARG for a NULL required pointer, B, Hq, Hkv, L,
  * per < 1, Hq % Hkv != 0, pos0 < 0 or pos0 + per > L, n_seeds < 0 or > L, or a
- * misaligned pointer; COVER_ERR_UNSUPPORTED for D != 128; COVER_ERR_CUDA for a
- * launch failure; COVER_ERR_DEVICE_TIMEOUT via cover_device_status.
+ * misaligned pointer; COVER_ERR_UNSUPPORTED for D != 128 or per > 16384 (the
+ * per-column data of a response block is staged in shared memory);
+ * COVER_ERR_CUDA for a launch failure; COVER_ERR_DEVICE_TIMEOUT via
+ * cover_device_status.
  */
 size_t cover_attn_mass_workspace_bytes(int B, int Hq, int per);
 int cover_attn_mass_fwd(const void* q, const void* k_cached, const void* k_seedmask,

@@ -287,7 +287,7 @@ int cover_attn_mass_fwd(const void* q, const void* k_cached, const void* k_seedm
       !aligned(tok, 4) || !aligned(d_in, 4) || !aligned(d_out, 4))
     return COVER_ERR_INVALID_ARG;
   if (n_seeds > 0 && (!aligned(k_seedmask, 16) || !aligned(seed_idx, 4))) return COVER_ERR_INVALID_ARG;
-  if (D != 128) return COVER_ERR_UNSUPPORTED;
+  if (D != 128 || per > cover::kMassMaxPer) return COVER_ERR_UNSUPPORTED;
   int* st = status_block();
   if (st == nullptr) return COVER_ERR_CUDA;
   cover::MassArgs a{q, k_cached, k_seedmask, seed_idx, n_seeds, lse, B, Hq, Hkv, L, pos0, per, tok, flags,

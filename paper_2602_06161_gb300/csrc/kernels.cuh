@@ -103,6 +103,7 @@ struct MassArgs {
   float* d_in;               // [B * per]
   float* d_out;              // [B * per]
 };
+constexpr int kMassMaxPer = 16384;   // a response block's per-column data is staged in shared memory
 size_t mass_workspace_bytes(int B, int Hq, int per);
 int launch_attn_mass(const MassArgs& a, int* status, cudaStream_t stream);
 

@@ -51,7 +51,7 @@ constexpr int kTmaWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kTileBytes = kT * kD * 2;     // 32 KB
 constexpr int kBoxBytes = kTileBytes / 2;   // one 64-column, 128-byte-swizzled box
-constexpr int kMaxPer = 16384;              // per-column staging must fit in shared memory
+constexpr int kMaxPer = kMassMaxPer;        // per-column staging must fit in shared memory
 
 // 128-byte aligned, so the per-column arrays that follow it start 16-byte aligned (float4 reads)
 struct alignas(128) MassSmem {

@@ -194,3 +194,9 @@ def test_mass_invalid_args(lib, kw):
 
 def test_mass_unsupported_head_dim(lib):
     assert lib.cover_attn_mass_fwd(P, P, P, P, 2, P, 1, 4, 2, 16, 64, P, P, 9, 8, 8, P, P, P, None) == -2
+
+
+def test_mass_unsupported_block_length(lib):
+    # a response block longer than the shared-memory staging holds
+    L = 20000
+    assert lib.cover_attn_mass_fwd(P, P, P, P, 2, P, 1, 4, 2, L, 128, P, P, 9, 0, 16385, P, P, P, None) == -2
