@@ -566,12 +566,14 @@ def prefix_timing(api, torch, q, kc, vc, km, vm, seeds, Lq, peak, hbm_gbs, iters
 
     A short window reads the whole memory of every head once for few query rows, so its bound is
     HBM: the line reports GB/s of algorithmic bytes (q and out of the window, K' and V', the
-    masked seed rows, the seed list and lse) beside the tensor-core fraction.
+    masked rows of the seeds inside the window - a seed outside it only overrides the memory, its
+    masked pair is never read - the seed list and lse) beside the tensor-core fraction.
     """
     B, Hq, L, D = q.shape
     Hkv = kc.shape[1]
     S = 0 if seeds is None else seeds.shape[1]
     q0 = L - Lq
+    s_in = 0 if seeds is None else int(((seeds >= q0) & (seeds < L)).sum().item())   # over all batch rows
     qw = q[:, :, q0:].contiguous()
     out = torch.empty_like(qw)
     lse = torch.empty((B, Hq, Lq), dtype=torch.float32, device=q.device)
@@ -589,7 +591,7 @@ def prefix_timing(api, torch, q, kc, vc, km, vm, seeds, Lq, peak, hbm_gbs, iters
         ts.append(a.elapsed_time(b))
     t = statistics.median(ts)
     flops = 4.0 * B * Hq * Lq * L * D
-    nbytes = 2 * (2 * B * Hq * Lq * D) + 2 * (2 * B * Hkv * L * D) + 2 * (2 * B * Hkv * S * D) + 4 * B * S \
+    nbytes = 2 * (2 * B * Hq * Lq * D) + 2 * (2 * B * Hkv * L * D) + 2 * (2 * Hkv * s_in * D) + 4 * B * S \
         + 4 * B * Hq * Lq
     gbs = nbytes / (t * 1e-3) / 1e9
     return {"Lq": Lq, "Lk": L, "q0": q0, "ms": round(t, 4), "tflops": round(flops / (t * 1e-3) / 1e12, 2),

@@ -555,9 +555,196 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
   }
 }
 
+// ---------------------------------------------------------------------------
+// Fast path of the per-segment work when the segment has at most one row per
+// thread of the CTA (per_seq <= blockDim.x): row i belongs to thread i, which
+// loads the row's state once (independent loads, one round trip to L2), keeps
+// it in registers and writes it back once. Each count takes one barrier
+// (__syncthreads_count). A top selection ranks every candidate against the
+// other candidates' keys in shared memory: its rank is the number of larger
+// keys, so the row of rank r < k is the (r+1)-th best and fills slot r. Keys
+// embed the row index, so they are distinct and the result is the general
+// path's (the sort or the rounds of maxima) exactly.
+// ---------------------------------------------------------------------------
+
+// Number of keys among keys[0 .. n) larger than x. All threads read the same
+// entry at the same time (shared-memory broadcasts).
+__device__ __forceinline__ int rank_of(const uint64_t* keys, int n, uint64_t x) {
+  int r = 0;
+#pragma unroll 4
+  for (int j = 0; j < n; ++j) r += keys[j] > x ? 1 : 0;
+  return r;
+}
+
+// Section 5.3 on the updated state, one row per thread (see segment_select for the
+// general path): seed score, n_t and the mean, n_t pi_t = #{n_t s_j > sum s}, and
+// the selection of ceil(sqrt(n_t pi_t)) rows by rank. Writes score, flags and the
+// segment's seed list, count and stats[4..5].
+__device__ void select_fast(uint64_t* keys, int seg, int per_seq, const DecideArgs& d, bool in, int tok,
+                            uint32_t& fl, uint32_t rc, float u, float din, float dout, float* score) {
+  __shared__ double s_sum[32];
+  __shared__ int s_elig;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+  const int n = seg * per_seq + tid;
+  float sc = -INFINITY;
+  bool valid = false;
+  uint64_t key = 0;
+  if (in && tok != d.mask_id) {
+    const float v = u * (1.0f + din) / (1.0f + dout);
+    if (isfinite(v)) {
+      sc = v;
+      valid = true;
+      if ((fl & 1u) == 0 && static_cast<int>(rc) < d.remask_budget) key = rank_key(v, tid);
+    }
+  }
+  double tot = valid ? static_cast<double>(sc) : 0.0;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+  const uint32_t eb = __ballot_sync(0xffffffffu, key != 0);
+  if (tid == 0) s_elig = 0;
+  if (lane == 0) s_sum[warp] = tot;
+  if (in) keys[tid] = key;
+  __syncthreads();
+  if (lane == 0 && eb != 0u) atomicAdd(&s_elig, __popc(eb));
+  const int n_t = __syncthreads_count(valid);
+  double total = 0.0;
+  for (int w = 0; w < nw; ++w) total += s_sum[w];
+  const int above = __syncthreads_count(valid && static_cast<double>(n_t) * static_cast<double>(sc) > total);
+  int k = 0;
+  while (k * k < above) ++k;   // ceil(sqrt(n_t pi_t))
+  k = min(k, d.max_seeds);
+  const int chosen = min(k, s_elig);
+  int slot = -1;
+  if (key != 0 && k > 0) {
+    const int r = rank_of(keys, per_seq, key);
+    if (r < k) slot = r;
+  }
+  if (in) {
+    score[n] = sc;
+    fl = (fl & ~3u) | (slot >= 0 ? 1u : 0u);
+  }
+  if (slot >= 0) d.seed_idx[static_cast<size_t>(seg) * d.max_seeds + slot] = d.pos0 + tid;
+  for (int t = chosen + tid; t < d.max_seeds; t += blockDim.x) d.seed_idx[static_cast<size_t>(seg) * d.max_seeds + t] = -1;
+  if (tid == 0) {
+    d.n_seeds[seg] = chosen;
+    if (d.stats != nullptr) {
+      int32_t* st = d.stats + static_cast<size_t>(seg) * kDecideStats;
+      st[4] = n_t;
+      st[5] = above;
+    }
+  }
+}
+
+// One segment's decision step, one row per thread (see segment_update and
+// segment_select for the general path).
+__device__ void decide_fast(uint64_t* keys, int seg, int per_seq, const ScoreParams& P) {
+  __shared__ unsigned long long s_fallback;
+  __shared__ int s_cnt[3];
+  __threadfence();
+  const DecideArgs& d = P.dec;
+  const int tid = threadIdx.x, lane = tid & 31;
+  const bool in = tid < per_seq;
+  const int n = seg * per_seq + tid;
+  const bool select = d.phase == 0;
+  // the row's whole state, in one round trip (other CTAs' results through L2)
+  int tok = 0, yhat = 0;
+  uint32_t fl = 0, rc = 0;
+  float c = 0.0f, H = 0.0f, u = 0.0f, lnz = 0.0f, din = 0.0f, dout = 0.0f;
+  bool ok_draft = false;
+  if (in) {
+    tok = d.tok[n];
+    fl = d.flags[n];
+    rc = d.remask_cnt[n];
+    ok_draft = d.draft_ok == nullptr || d.draft_ok[n] != 0;
+    c = __ldcg(P.maxprob + n);
+    H = __ldcg(P.entropy + n);
+    yhat = __ldcg(P.argmax + n);
+    u = __ldcg(d.ws_u + n);
+    lnz = __ldcg(d.ws_lnz + n);
+    if (select) {
+      din = P.d_in != nullptr ? P.d_in[n] : 0.0f;
+      dout = P.d_out != nullptr ? P.d_out[n] : 0.0f;
+    }
+  }
+  if (tid == 0) {
+    s_fallback = ~0ull;
+    s_cnt[0] = s_cnt[1] = s_cnt[2] = 0;
+  }
+  __syncthreads();
+
+  // Section 5.2 drafting: masked rows in the allowed set whose confidence exceeds tau
+  const bool allowed = in && tok == d.mask_id && ok_draft;
+  const bool cand = allowed && c > d.tau;
+  if (d.min_one && allowed)   // lowest entropy, then lowest index
+    atomicMin(&s_fallback, static_cast<unsigned long long>((static_cast<uint64_t>(order_key(H)) << 32) |
+                                                            static_cast<uint32_t>(tid)));
+  const int ncand = __syncthreads_count(cand);
+  const bool all_cand = ncand <= d.budget;   // every row above tau is drafted
+  int n_drafted = min(ncand, d.budget);
+  bool drafted = all_cand && cand;
+  if (!all_cand) {
+    // more candidates than the budget: the `budget` most confident (ties to the lower index)
+    if (in) keys[tid] = cand ? rank_key(c, tid) : 0ull;
+    __syncthreads();
+    if (cand) drafted = rank_of(keys, per_seq, rank_key(c, tid)) < d.budget;
+    __syncthreads();   // the keys are rewritten by the selection
+  }
+  if (n_drafted == 0 && d.min_one && s_fallback != ~0ull) {
+    n_drafted = 1;
+    drafted = in && tid == static_cast<int>(static_cast<uint32_t>(s_fallback));
+  }
+
+  // Section 5.2 revision of the previous seeds, Section 3 state update
+  bool kept = false, replaced = false, remasked = false;
+  if (drafted) {
+    // a drafted row takes its greedy token, whose uncertainty is ln Z
+    tok = yhat;
+    u = lnz;
+    fl = (fl & ~1u) | 2u;
+  } else if (in && (fl & 1u) != 0 && tok != d.mask_id) {
+    if (yhat == tok) {
+      kept = true;
+    } else if (c > d.tau) {
+      replaced = true;
+      tok = yhat;
+      u = lnz;
+    } else {
+      remasked = true;
+      tok = d.mask_id;
+      rc = min(rc + 1u, 255u);
+    }
+  }
+  const uint32_t bk = __ballot_sync(0xffffffffu, kept), br = __ballot_sync(0xffffffffu, replaced),
+                 bm = __ballot_sync(0xffffffffu, remasked);
+  if (lane == 0) {
+    if (bk) atomicAdd(&s_cnt[0], __popc(bk));
+    if (br) atomicAdd(&s_cnt[1], __popc(br));
+    if (bm) atomicAdd(&s_cnt[2], __popc(bm));
+  }
+  if (select) select_fast(keys, seg, per_seq, d, in, tok, fl, rc, u, din, dout, P.score);
+  else __syncthreads();
+  if (in) {
+    d.tok[n] = tok;
+    d.flags[n] = static_cast<uint8_t>(fl);
+    d.remask_cnt[n] = static_cast<uint8_t>(rc);
+    d.ws_u[n] = u;
+  }
+  if (tid == 0 && d.stats != nullptr) {
+    int32_t* st = d.stats + static_cast<size_t>(seg) * kDecideStats;
+    st[0] = n_drafted;
+    st[1] = s_cnt[0];
+    st[2] = s_cnt[1];
+    st[3] = s_cnt[2];
+  }
+}
+
 // The last CTA of a segment in decision mode: the update, then (unless only the
 // update was asked for) the selection with the caller's d_in / d_out.
 __device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n, const ScoreParams& P) {
+  if (per_seq <= static_cast<int>(blockDim.x)) {
+    decide_fast(keys, seg, per_seq, P);
+    return;
+  }
   segment_update(keys, seg, per_seq, sort_n, P);
   if (P.dec.phase == 0) {
     __syncthreads();
@@ -572,6 +759,29 @@ __device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_se
   __threadfence();
   const int tid = threadIdx.x, nt = blockDim.x;
   const int base = seg * per_seq;
+  if (per_seq <= nt) {
+    // one row per thread: rank every eligible row against the others (see decide_fast)
+    uint64_t key = 0;
+    float sc = 0.0f;
+    if (tid < per_seq && (eligible == nullptr || eligible[base + tid] != 0)) {
+      sc = __ldcg(score + base + tid);
+      key = rank_key(sc, tid);
+    }
+    if (tid < per_seq) keys[tid] = key;
+    const int n_elig = __syncthreads_count(key != 0);
+    if (key != 0) {
+      const int r = rank_of(keys, per_seq, key);
+      if (r < topk) {
+        topk_idx[static_cast<size_t>(seg) * topk + r] = tid;
+        if (topk_score != nullptr) topk_score[static_cast<size_t>(seg) * topk + r] = sc;
+      }
+    }
+    for (int t = min(n_elig, topk) + tid; t < topk; t += nt) {
+      topk_idx[static_cast<size_t>(seg) * topk + t] = -1;
+      if (topk_score != nullptr) topk_score[static_cast<size_t>(seg) * topk + t] = -INFINITY;
+    }
+    return;
+  }
   for (int i = tid; i < sort_n; i += nt) {
     uint64_t key = 0;
     if (i < per_seq && (eligible == nullptr || eligible[base + i] != 0)) {
@@ -581,9 +791,18 @@ __device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_se
     keys[i] = key;
   }
   __syncthreads();
-  bitonic_sort_desc(keys, sort_n);
+  // a short list by rounds of maxima (one barrier each), a long one by sorting
+  __shared__ unsigned long long s_top[2][32];
+  __shared__ uint64_t s_sel[kRoundsMax];
+  const uint64_t* best = keys;
+  if (topk <= kRoundsMax) {
+    top_rounds(keys, sort_n, topk, s_sel, s_top);
+    best = s_sel;
+  } else {
+    bitonic_sort_desc(keys, sort_n);
+  }
   for (int t = tid; t < topk; t += nt) {
-    const uint64_t key = keys[t];
+    const uint64_t key = best[t];
     const bool valid = key != 0;
     topk_idx[static_cast<size_t>(seg) * topk + t] =
         valid ? static_cast<int32_t>(0xffffffffu - static_cast<uint32_t>(key)) : -1;
@@ -801,6 +1020,26 @@ __global__ void __launch_bounds__(kSelectThreads) seed_select_kernel(const Decid
                                                                     const float* d_out, float* score, int per_seq,
                                                                     int sort_n) {
   extern __shared__ uint64_t sel_keys[];
+  const int tid = threadIdx.x;
+  if (per_seq <= static_cast<int>(blockDim.x)) {
+    // one row per thread: the state in registers, selection by rank
+    const int n = blockIdx.x * per_seq + tid;
+    const bool in = tid < per_seq;
+    int tok = 0;
+    uint32_t fl = 0, rc = 0;
+    float u = 0.0f, din = 0.0f, dout = 0.0f;
+    if (in) {
+      tok = d.tok[n];
+      fl = d.flags[n];
+      rc = d.remask_cnt[n];
+      u = d.ws_u[n];
+      din = d_in != nullptr ? d_in[n] : 0.0f;
+      dout = d_out != nullptr ? d_out[n] : 0.0f;
+    }
+    select_fast(sel_keys, blockIdx.x, per_seq, d, in, tok, fl, rc, u, din, dout, score);
+    if (in) d.flags[n] = static_cast<uint8_t>(fl);
+    return;
+  }
   segment_select(sel_keys, blockIdx.x, per_seq, sort_n, d, d_in, d_out, score);
 }
 
