@@ -152,6 +152,13 @@ __global__ void __launch_bounds__(kThreads, 2)
     tmem_relinquish();
   }
   route_clear(sm.slot, kT, tid, kThreads);
+  // the first seed entry of this thread, loaded now so that its latency overlaps the column data's
+  const int32_t* seeds_b = seed_idx + static_cast<size_t>(b) * n_seeds;
+  const int seed0 = tid < n_seeds ? __ldg(seeds_b + tid) : -1;
+  // rows CTAs: the log2-scaled lse of the thread's own query (thread = row of the tile)
+  float own = 0.0f;
+  if (!cols && tid < kMathThreads && t * kT + tid < per)
+    own = lse[static_cast<size_t>(bh) * L + pos0 + t * kT + tid] * 1.4426950408889634f;
   // per-column data of the whole block: rows CTAs need the drafted keys, columns CTAs the masked
   // queries and their lse; one warp per 32 columns
   for (int w = warp; w < n_t * 4; w += kThreads / 32) {
@@ -171,7 +178,15 @@ __global__ void __launch_bounds__(kThreads, 2)
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
-  route_scan(sm.slot, seed_idx + static_cast<size_t>(b) * n_seeds, n_seeds, pos0 + t * kT, kT, L, tid, kThreads);
+  {
+    // seed routing of the resident tile's positions (the lowest slot naming a position wins)
+    const int row0 = pos0 + t * kT;
+    if (seed0 >= row0 && seed0 < row0 + kT && seed0 < L) atomicMin(sm.slot + (seed0 - row0), tid);
+    for (int sidx = tid + kThreads; sidx < n_seeds; sidx += kThreads) {
+      const int p = __ldg(seeds_b + sidx);
+      if (p >= row0 && p < row0 + kT && p < L) atomicMin(sm.slot + (p - row0), sidx);
+    }
+  }
   __syncthreads();
   const uint32_t tbase = sm.tmem_base;
 
@@ -238,8 +253,6 @@ __global__ void __launch_bounds__(kThreads, 2)
     const size_t qrow = (static_cast<size_t>(bh) * L + pos0 + i) * kD;
     // the diagonal entry of a seed query uses its masked-input key (leave-one-out view)
     const int my_slot = valid ? sm.slot[r] : kNoSlot;
-    float own = 0.0f;                                  // rows: lse of the thread's query; columns: unused
-    if (!cols && valid) own = lse[static_cast<size_t>(bh) * L + pos0 + i] * 1.4426950408889634f;
     float p_self = 0.0f;
     if (my_slot != kNoSlot) {
       const float lse2 = cols ? colv[i] : own;         // +inf for a query that is not masked: weight 0

@@ -933,13 +933,21 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
   const int nchunks = (V + kChunkElems - 1) / kChunkElems;
   uint8_t* ring = dsmem;
 
-  if (tid == 0) {
+  if (warp == kConsumerWarps && lane == 0) {
+    // the producer initialises the ring and issues its first chunks at once, so their latency
+    // overlaps the block barrier
     for (int s = 0; s < kRingStages; ++s) {
       mbar_init(&bar_full[s], 1);
       mbar_init(&bar_empty[s], kConsumerWarps);
     }
     s_abort = 0;
     fence_mbar_init();
+    for (int c = 0; c < kRingStages && c < nchunks; ++c) {
+      const int elems = min(kChunkElems, V - c * kChunkElems);
+      mbar_arrive_expect_tx(&bar_full[c], static_cast<uint32_t>(elems * 2));
+      bulk_load(ring + c * kChunkBytes, row + static_cast<size_t>(c) * kChunkElems, static_cast<uint32_t>(elems * 2),
+                &bar_full[c]);
+    }
   }
   __syncthreads();
 
@@ -947,9 +955,9 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
   if (warp == kConsumerWarps) {
     // producer: one lane streams the row chunk by chunk
     if (lane == 0) {
-      for (int c = 0; c < nchunks; ++c) {
+      for (int c = kRingStages; c < nchunks; ++c) {
         const int st = c % kRingStages;
-        if (c >= kRingStages && !mbar_wait(&bar_empty[st], ((c / kRingStages) - 1) & 1, &s_abort)) {
+        if (!mbar_wait(&bar_empty[st], ((c / kRingStages) - 1) & 1, &s_abort)) {
           report_status(status, kStatusTimeout, 200);
           s_abort = 1;
           break;
