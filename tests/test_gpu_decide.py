@@ -181,3 +181,57 @@ def test_decide_named_workload_full():
     rng = np.random.default_rng(0)
     rows = np.sort(rng.choice(di.N, size=128, replace=False))
     check(di, p, run_decide(di, p), fp64_rows=rows, what=wl.name)
+
+
+@pytest.mark.parametrize("per,V", [
+    (288, 1000),   # one row per thread of the bulk-copy kernel (288 threads): the fast path
+    (289, 1000),   # one row more than its threads: the general path
+    (512, 1001),   # the register-load kernel (odd vocabulary, 512 threads): its fast-path limit
+    (513, 1001),   # and one row past it
+])
+def test_decide_both_sides_of_the_fast_path(per, V):
+    # the per-sequence decision has a one-row-per-thread path and a general one; on both sides
+    # of the switch the decisions equal the oracle's, with a drafting budget that forces the
+    # ranking (more candidates than the budget) and a seed cap above 32 (sort instead of rounds)
+    di = W.make_decide_inputs(2 * per, V, 2, seed=per, block_len=64)
+    for p in (_params(draft_budget=15, max_seeds=8), _params(draft_budget=2, tau_draft=0.05, max_seeds=40)):
+        check(di, p, run_decide(di, p), what=f"per {per} V {V} B {p['draft_budget']}")
+
+
+@pytest.mark.parametrize("per", [256, 512, 513, 1024])
+def test_update_then_select_both_paths(per):
+    # the split order (update phase, then the selection launch with the caller's d_in / d_out):
+    # the selection launch has 512 threads, so 512 rows take its fast path and 513 the general one
+    di = W.make_decide_inputs(2 * per, 1000, 2, seed=per + 1, block_len=32)
+    p = _params(max_seeds=12)
+    logits = H.to_dev(di.logits, "bf16")
+    tok = torch.from_numpy(di.tok.copy()).cuda()
+    flags = torch.from_numpy(di.flags.copy()).cuda()
+    rc = torch.from_numpy(di.remask_cnt.copy()).cuda()
+    ws = api.decide_workspace(di.N, di.n_seq)
+    kw = dict(tau_draft=p["tau_draft"], draft_budget=p["draft_budget"], remask_budget=p["remask_budget"],
+              mask_id=di.mask_id, min_one=p["min_one"], pos0=p["pos0"], max_seeds=p["max_seeds"])
+    upd = api.cover_score_decide_fwd(logits, di.n_seq, tok, flags, rc, phase=api.COVER_DECIDE_UPDATE,
+                                     workspace=ws, draft_ok=torch.from_numpy(di.draft_ok).cuda(), **kw)
+    d_in, d_out = H.to_dev(di.d_in, "f32"), H.to_dev(di.d_out, "f32")
+    sel = api.cover_seed_select_fwd(di.n_seq, tok, flags, rc, ws, remask_budget=p["remask_budget"],
+                                    mask_id=di.mask_id, pos0=p["pos0"], max_seeds=p["max_seeds"], d_in=d_in,
+                                    d_out=d_out)
+    torch.cuda.synchronize()
+    assert api.cover_device_status() == 0
+    u_cur = api.cover_score_fwd(logits, di.n_seq, 0, cur_tok=torch.from_numpy(di.tok).cuda())["score"].cpu().numpy()
+    u_top = api.cover_score_fwd(logits, di.n_seq, 0)["score"].cpu().numpy()
+    h = {k: v.cpu().numpy() for k, v in upd.items()}
+    outs = oracle.decide_step(h["maxprob"], h["argmax"], h["entropy"], u_cur, u_top, di.d_in, di.d_out, di.tok,
+                              di.flags, di.remask_cnt, di.draft_ok, di.n_seq, tau=F32(p["tau_draft"]),
+                              budget=p["draft_budget"], m_remask=p["remask_budget"], mask_id=di.mask_id,
+                              min_one=p["min_one"], pos0=p["pos0"], max_seeds=p["max_seeds"])
+    t, fl, r_, sc = tok.cpu().numpy(), flags.cpu().numpy(), rc.cpu().numpy(), sel["score"].cpu().numpy()
+    for g, o in enumerate(outs):
+        sl = slice(g * per, (g + 1) * per)
+        assert np.array_equal(t[sl], o["tok"]) and np.array_equal(r_[sl], o["remask_cnt"]), (per, g)
+        assert np.array_equal(fl[sl], o["flags"]), (per, g)
+        assert np.array_equal(sc[sl], o["score"].astype(F32)), (per, g)
+        seeds = o["seeds"] + [-1] * (p["max_seeds"] - len(o["seeds"]))
+        assert sel["seed_idx"][g].cpu().tolist() == seeds, (per, g)
+        assert int(sel["n_seeds"][g]) == o["n_select"], (per, g)

@@ -98,3 +98,15 @@ def test_score_named_workloads_full(name):
     ref = check(inp, r, name)
     gaps = oracle.topk_margin(ref["score"], inp.n_seq, inp.topk)
     print(f"{name}: top-k margins min {gaps.min():.3e}")
+
+
+@pytest.mark.parametrize("per,V,k", [
+    (288, 1000, 40),    # one row per thread of the bulk-copy kernel: selection by rank
+    (289, 1000, 20),    # the general path, a short list: rounds of maxima
+    (289, 1000, 40),    # the general path, a long list: the bitonic sort
+    (512, 1001, 33),    # the register-load kernel (512 threads): selection by rank
+    (513, 1001, 32),    # and one row past it: rounds of maxima
+])
+def test_score_topk_on_both_sides_of_the_fast_path(per, V, k):
+    inp = W.make_score_inputs(2 * per, V, 2, k, seed=per + k, spike_frac=0.1, eligible_frac=0.8)
+    check(inp, run_score(inp), f"per {per} V {V} k {k}")
