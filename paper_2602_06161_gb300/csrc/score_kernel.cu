@@ -567,12 +567,23 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
 // path's (the sort or the rounds of maxima) exactly.
 // ---------------------------------------------------------------------------
 
-// Number of keys among keys[0 .. n) larger than x. All threads read the same
-// entry at the same time (shared-memory broadcasts).
-__device__ __forceinline__ int rank_of(const uint64_t* keys, int n, uint64_t x) {
-  int r = 0;
-#pragma unroll 4
-  for (int j = 0; j < n; ++j) r += keys[j] > x ? 1 : 0;
+// Rank of x among keys[0 .. n) (16-byte aligned): the number of larger keys, counted only while
+// it can still be below k. All threads read the same entries at the same time (shared-memory
+// broadcasts, two keys per load); a warp stops once every lane's count has reached k (x = 0,
+// no key, counts as already there), and the result is then some value >= k.
+__device__ __forceinline__ int rank_below(const uint64_t* keys, int n, uint64_t x, int k) {
+  int r = x != 0 ? 0 : k;
+  const ulonglong2* k2 = reinterpret_cast<const ulonglong2*>(keys);
+  int j = 0;
+  for (; j + 32 <= n; j += 32) {
+    if (__all_sync(0xffffffffu, r >= k)) return r;
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      const ulonglong2 y = k2[(j >> 1) + q];
+      r += (y.x > x ? 1 : 0) + (y.y > x ? 1 : 0);
+    }
+  }
+  for (; j < n; ++j) r += keys[j] > x ? 1 : 0;
   return r;
 }
 
@@ -582,7 +593,8 @@ __device__ __forceinline__ int rank_of(const uint64_t* keys, int n, uint64_t x) 
 // segment's seed list, count and stats[4..5].
 __device__ void select_fast(uint64_t* keys, int seg, int per_seq, const DecideArgs& d, bool in, int tok,
                             uint32_t& fl, uint32_t rc, float u, float din, float dout, float* score) {
-  __shared__ double s_sum[32];
+  __shared__ long long s_fx[32];
+  __shared__ uint32_t s_emax;
   __shared__ int s_elig;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
   const int n = seg * per_seq + tid;
@@ -597,27 +609,52 @@ __device__ void select_fast(uint64_t* keys, int seg, int per_seq, const DecideAr
       if ((fl & 1u) == 0 && static_cast<int>(rc) < d.remask_budget) key = rank_key(v, tid);
     }
   }
-  double tot = valid ? static_cast<double>(sc) : 0.0;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+  // n_t pi_t = #{n_t s_j > sum s} in exact integer arithmetic. Every score becomes a 64-bit
+  // fixed-point integer on the sequence's largest binade: S = s 2^(26 - E) with E the largest
+  // exponent, so |S| < 2^50, exact for every score within a factor 2^26 of the largest (a smaller
+  // one is truncated toward zero; it lies far below the mean, and the sum's error stays below
+  // n_t units, 2^-50 of the largest score). The sum and the products n_t S (|n_t S| < 2^62) are
+  // exact integers; this GPU's fp64 units have long latencies, so no fp64 is used here.
+  const uint32_t sbits = __float_as_uint(sc);
+  const uint32_t ebias = valid ? ((sbits >> 23) & 0xffu) : 0u;
+  const uint32_t emax_w = __reduce_max_sync(0xffffffffu, ebias);
   const uint32_t eb = __ballot_sync(0xffffffffu, key != 0);
-  if (tid == 0) s_elig = 0;
-  if (lane == 0) s_sum[warp] = tot;
+  if (tid == 0) {
+    s_elig = 0;
+    s_emax = 0u;
+  }
   if (in) keys[tid] = key;
   __syncthreads();
-  if (lane == 0 && eb != 0u) atomicAdd(&s_elig, __popc(eb));
+  if (lane == 0) {
+    atomicMax(&s_emax, emax_w);
+    if (eb != 0u) atomicAdd(&s_elig, __popc(eb));
+  }
   const int n_t = __syncthreads_count(valid);
-  double total = 0.0;
-  for (int w = 0; w < nw; ++w) total += s_sum[w];
-  const int above = __syncthreads_count(valid && static_cast<double>(n_t) * static_cast<double>(sc) > total);
+  long long fx = 0;
+  if (valid) {
+    // s = m 2^(ebias - 150) (m with its leading bit; a denormal has ebias 0 and exponent 1 - 150)
+    const uint32_t m = ebias != 0u ? ((sbits & 0x7fffffu) | 0x800000u) : (sbits & 0x7fffffu);
+    const int shift = static_cast<int>(ebias == 0u ? 1u : ebias) - static_cast<int>(s_emax) + 26;
+    const long long mag = shift >= 0 ? (static_cast<long long>(m) << shift) : (shift > -25 ? (m >> -shift) : 0);
+    fx = (sbits >> 31) ? -mag : mag;
+  }
+  long long tot = fx;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+  if (lane == 0) s_fx[warp] = tot;
+  __syncthreads();
+  long long total = 0;
+  for (int w = 0; w < nw; ++w) total += s_fx[w];
+  const bool is_above = valid && static_cast<long long>(n_t) * fx > total;
+  const int above = __syncthreads_count(is_above);
   int k = 0;
   while (k * k < above) ++k;   // ceil(sqrt(n_t pi_t))
   k = min(k, d.max_seeds);
   const int chosen = min(k, s_elig);
   int slot = -1;
-  if (key != 0 && k > 0) {
-    const int r = rank_of(keys, per_seq, key);
-    if (r < k) slot = r;
+  if (k > 0) {
+    const int r = rank_below(keys, per_seq, key, k);
+    if (key != 0 && r < k) slot = r;
   }
   if (in) {
     score[n] = sc;
@@ -686,7 +723,7 @@ __device__ void decide_fast(uint64_t* keys, int seg, int per_seq, const ScorePar
     // more candidates than the budget: the `budget` most confident (ties to the lower index)
     if (in) keys[tid] = cand ? rank_key(c, tid) : 0ull;
     __syncthreads();
-    if (cand) drafted = rank_of(keys, per_seq, rank_key(c, tid)) < d.budget;
+    drafted = rank_below(keys, per_seq, cand ? rank_key(c, tid) : 0ull, d.budget) < d.budget && cand;
     __syncthreads();   // the keys are rewritten by the selection
   }
   if (n_drafted == 0 && d.min_one && s_fallback != ~0ull) {
@@ -769,9 +806,9 @@ __device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_se
     }
     if (tid < per_seq) keys[tid] = key;
     const int n_elig = __syncthreads_count(key != 0);
-    if (key != 0) {
-      const int r = rank_of(keys, per_seq, key);
-      if (r < topk) {
+    {
+      const int r = rank_below(keys, per_seq, key, topk);
+      if (key != 0 && r < topk) {
         topk_idx[static_cast<size_t>(seg) * topk + r] = tid;
         if (topk_score != nullptr) topk_score[static_cast<size_t>(seg) * topk + r] = sc;
       }
@@ -861,7 +898,7 @@ __device__ __forceinline__ void acc_batch(RowAcc& a, const uint4 (&w)[U], int i0
 // register-load kernel (any V)
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads, 2) score_kernel(const ScoreParams P) {
-  extern __shared__ uint64_t keys[];
+  extern __shared__ __align__(16) uint64_t keys[];
   __shared__ float red_m[kWarps];
   __shared__ int red_i[kWarps];
   __shared__ double red_z[kWarps], red_s[kWarps];
@@ -1027,7 +1064,7 @@ constexpr int kSelectThreads = 512;
 __global__ void __launch_bounds__(kSelectThreads) seed_select_kernel(const DecideArgs d, const float* d_in,
                                                                     const float* d_out, float* score, int per_seq,
                                                                     int sort_n) {
-  extern __shared__ uint64_t sel_keys[];
+  extern __shared__ __align__(16) uint64_t sel_keys[];
   const int tid = threadIdx.x;
   if (per_seq <= static_cast<int>(blockDim.x)) {
     // one row per thread: the state in registers, selection by rank
