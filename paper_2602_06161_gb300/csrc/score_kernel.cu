@@ -587,6 +587,42 @@ __device__ __forceinline__ int rank_below(const uint64_t* keys, int n, uint64_t 
   return r;
 }
 
+// Descending bitonic sort of a warp's 32 keys, one per lane, by shuffles.
+__device__ __forceinline__ uint64_t warp_sort_desc(uint64_t key, int lane) {
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1) {
+    const bool desc = (lane & size) == 0;
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const uint64_t other = __shfl_xor_sync(0xffffffffu, key, stride);
+      const bool take_max = ((lane & stride) == 0) == desc;
+      key = take_max ? (key > other ? key : other) : (key < other ? key : other);
+    }
+  }
+  return key;
+}
+
+// The k largest (k <= 32) of the CTA's keys, one per thread (distinct, 0 = none). Each warp sorts
+// its keys and publishes its k largest in cand[warp * k ..]; a key can be among the CTA's k
+// largest only if it is among its warp's, and the number of larger published keys is its rank,
+// exact while below k (a warp publishes at most k). Returns, for the key this lane holds after
+// its warp's sort (*held), its slot 0 .. k-1 among the CTA's k largest, else -1. All threads of
+// the CTA call it; cand holds blockDim.x keys.
+__device__ __forceinline__ int top_small(uint64_t key, int k, uint64_t* cand, uint64_t* held) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const uint64_t sorted = warp_sort_desc(key, lane);
+  if (lane < k) cand[warp * k + lane] = sorted;
+  __syncthreads();
+  int slot = -1;
+  if (lane < k && sorted != 0) {
+    int r = 0;
+    for (int j = 0; j < nw * k; ++j) r += cand[j] > sorted ? 1 : 0;
+    if (r < k) slot = r;
+  }
+  *held = sorted;
+  return slot;
+}
+
 // Section 5.3 on the updated state, one row per thread (see segment_select for the
 // general path): seed score, n_t and the mean, n_t pi_t = #{n_t s_j > sum s}, and
 // the selection of ceil(sqrt(n_t pi_t)) rows by rank. Writes score, flags and the
@@ -596,6 +632,7 @@ __device__ void select_fast(uint64_t* keys, int seg, int per_seq, const DecideAr
   __shared__ long long s_fx[32];
   __shared__ uint32_t s_emax;
   __shared__ int s_elig;
+  __shared__ uint8_t s_mark[512];   // blockDim <= 512
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
   const int n = seg * per_seq + tid;
   float sc = -INFINITY;
@@ -651,16 +688,31 @@ __device__ void select_fast(uint64_t* keys, int seg, int per_seq, const DecideAr
   while (k * k < above) ++k;   // ceil(sqrt(n_t pi_t))
   k = min(k, d.max_seeds);
   const int chosen = min(k, s_elig);
-  int slot = -1;
-  if (k > 0) {
+  bool chosen_row = false;
+  if (k > 0 && k <= 32) {
+    // few seeds: per-warp sorts and the ranks of the published keys; the lane holding a chosen
+    // key writes its slot and marks the row for its owner thread
+    uint64_t held;
+    if (in) s_mark[tid] = 0;
+    const int slot = top_small(key, k, keys, &held);
+    if (slot >= 0) {
+      const int row = rank_key_row(held);
+      d.seed_idx[static_cast<size_t>(seg) * d.max_seeds + slot] = d.pos0 + row;
+      s_mark[row] = 1;
+    }
+    __syncthreads();
+    chosen_row = in && s_mark[tid] != 0;
+  } else if (k > 0) {
     const int r = rank_below(keys, per_seq, key, k);
-    if (key != 0 && r < k) slot = r;
+    if (key != 0 && r < k) {
+      chosen_row = true;
+      d.seed_idx[static_cast<size_t>(seg) * d.max_seeds + r] = d.pos0 + tid;
+    }
   }
   if (in) {
     score[n] = sc;
-    fl = (fl & ~3u) | (slot >= 0 ? 1u : 0u);
+    fl = (fl & ~3u) | (chosen_row ? 1u : 0u);
   }
-  if (slot >= 0) d.seed_idx[static_cast<size_t>(seg) * d.max_seeds + slot] = d.pos0 + tid;
   for (int t = chosen + tid; t < d.max_seeds; t += blockDim.x) d.seed_idx[static_cast<size_t>(seg) * d.max_seeds + t] = -1;
   if (tid == 0) {
     d.n_seeds[seg] = chosen;
@@ -677,6 +729,7 @@ __device__ void select_fast(uint64_t* keys, int seg, int per_seq, const DecideAr
 __device__ void decide_fast(uint64_t* keys, int seg, int per_seq, const ScoreParams& P) {
   __shared__ unsigned long long s_fallback;
   __shared__ int s_cnt[3];
+  __shared__ uint8_t s_draft[512];   // blockDim <= 512
   __threadfence();
   const DecideArgs& d = P.dec;
   const int tid = threadIdx.x, lane = tid & 31;
@@ -721,9 +774,19 @@ __device__ void decide_fast(uint64_t* keys, int seg, int per_seq, const ScorePar
   bool drafted = all_cand && cand;
   if (!all_cand) {
     // more candidates than the budget: the `budget` most confident (ties to the lower index)
-    if (in) keys[tid] = cand ? rank_key(c, tid) : 0ull;
-    __syncthreads();
-    drafted = rank_below(keys, per_seq, cand ? rank_key(c, tid) : 0ull, d.budget) < d.budget && cand;
+    const uint64_t ck = cand ? rank_key(c, tid) : 0ull;
+    if (d.budget <= 32) {
+      if (in) s_draft[tid] = 0;
+      uint64_t held;
+      const int slot = top_small(ck, d.budget, keys, &held);
+      if (slot >= 0) s_draft[rank_key_row(held)] = 1;
+      __syncthreads();
+      drafted = in && s_draft[tid] != 0;
+    } else {
+      if (in) keys[tid] = ck;
+      __syncthreads();
+      drafted = rank_below(keys, per_seq, ck, d.budget) < d.budget && cand;
+    }
     __syncthreads();   // the keys are rewritten by the selection
   }
   if (n_drafted == 0 && d.min_one && s_fallback != ~0ull) {
@@ -1099,9 +1162,12 @@ int launch_score_impl(const ScoreArgs& a, const DecideArgs* d, int* status, cuda
   ScoreParams P{static_cast<const uint16_t*>(a.logits), a.V, per, a.cur_tok, a.d_in, a.d_out, a.eligible,
                 a.topk, sort_n, a.maxprob, a.entropy, a.argmax, a.score, a.topk_idx, a.topk_score, a.counters,
                 d != nullptr ? 1 : 0, d != nullptr ? *d : DecideArgs{}};
-  // top-k keys; the decision step also keeps a float score per row behind them
-  const size_t keys_bytes = d != nullptr ? (sizeof(uint64_t) + sizeof(float)) * static_cast<size_t>(sort_n)
-                            : a.topk > 0 ? sizeof(uint64_t) * static_cast<size_t>(sort_n) : 0;
+  // top-k keys; the decision step also keeps a float score per row behind them. At least one key
+  // per thread of the register-load kernel: the one-row-per-thread selection publishes up to
+  // 32 keys per warp.
+  const size_t key_slots = static_cast<size_t>(std::max(sort_n, kThreads));
+  const size_t keys_bytes = d != nullptr ? (sizeof(uint64_t) + sizeof(float)) * key_slots
+                            : a.topk > 0 ? sizeof(uint64_t) * key_slots : 0;
   const bool aligned_rows = (a.V % 8) == 0 && (reinterpret_cast<uintptr_t>(a.logits) % 16) == 0;
   if (aligned_rows) {
     const size_t smem = std::max(keys_bytes, static_cast<size_t>(kRingStages) * kChunkBytes);
@@ -1135,7 +1201,8 @@ int launch_seed_select(int N, int n_seq, const DecideArgs& d, const float* d_in,
   const int per = N / n_seq;
   int sort_n = 1;
   while (sort_n < per) sort_n <<= 1;
-  const size_t smem = (sizeof(uint64_t) + sizeof(float)) * static_cast<size_t>(sort_n);
+  // at least one key per thread: the one-row-per-thread selection publishes up to 32 keys per warp
+  const size_t smem = (sizeof(uint64_t) + sizeof(float)) * static_cast<size_t>(std::max(sort_n, kSelectThreads));
   seed_select_kernel<<<n_seq, kSelectThreads, smem, stream>>>(d, d_in, d_out, score, per, sort_n);
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
