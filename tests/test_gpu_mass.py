@@ -73,6 +73,7 @@ def oracle_mass(inp, masked, drafted, pos0, batches=None):
     (1, 7, 1, 160, 5, 31, 129),       # GQA 7:1, one row past a tile
     (2, 2, 2, 64, 3, 63, 1),          # a single response position
     (1, 2, 2, 256, 0, 64, 192),       # no seeds
+    (1, 4, 2, 1100, 10, 460, 640),    # five tiles each way: the two-stage rings wrap twice
 ])
 def test_mass_against_oracle(B, Hq, Hkv, L, S, pos0, per):
     inp = W.make_attn_inputs(B, Hq, Hkv, L, 128, S, dtype="bf16", seed=L + per, seed_lo=0, seed_hi=L)
