@@ -8,8 +8,8 @@
 // with p = softmax(logits) at temperature 1. Each thread keeps, for its share
 // of the row, the running maximum m (exact bf16 compare, first index kept),
 // Z = sum 2^t and S = sum t 2^t with t = x log2(e) - m log2(e), Kahan
-// compensated; partials are re-referenced to the row maximum, summed across
-// each warp in fp32 with error-free TwoSum pairs and across warps in fp64.
+// compensated; partials are re-referenced to the row maximum and summed across
+// the warp and then across the warps in fp32 with error-free TwoSum pairs.
 // Then c = 1/Z, H = ln Z - ln(2) S / Z, u = ln Z - (x_y - m).
 //
 // Top-k (Section 5.3): the last CTA to finish a segment (sequence) - found
@@ -131,12 +131,20 @@ __device__ __forceinline__ float order_key_inv(uint32_t k) {
 struct RowOut {
   float M;      // row maximum
   int yhat;     // first index attaining it
-  double Z, S;  // sum 2^t and sum t 2^t re-referenced to M log2(e)
+  float Z;      // sum 2^t re-referenced to M log2(e)
+  float q;      // (sum t 2^t) / Z
 };
 
+// a + b = s + e exactly (Knuth's TwoSum)
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+  s = a + b;
+  const float bb = s - a;
+  e = (a - (s - bb)) + (b - bb);
+}
+
 template <int NW>
-__device__ __forceinline__ RowOut row_reduce(const RowAcc& a, float* red_m, int* red_i, double* red_z,
-                                             double* red_s) {
+__device__ __forceinline__ RowOut row_reduce(const RowAcc& a, float* red_m, int* red_i, float2* red_z,
+                                             float2* red_s) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   float m = a.m;
   int mi = a.mi;
@@ -167,8 +175,8 @@ __device__ __forceinline__ RowOut row_reduce(const RowAcc& a, float* red_m, int*
   }
   const float Mref = M * kLog2e;
   // partials re-referenced to the row maximum, summed across the warp in fp32
-  // with error-free TwoSum pairs (value, rounding error); fp64 only for the
-  // final sum of the per-warp results
+  // with error-free TwoSum pairs (value, rounding error), then across the warps
+  // the same way by thread 0
   float z = 0.0f, ze = 0.0f, sv = 0.0f, se = 0.0f;
   if (a.m != -INFINITY) {
     const float d = a.mref - Mref;
@@ -191,16 +199,31 @@ __device__ __forceinline__ RowOut row_reduce(const RowAcc& a, float* red_m, int*
     sv = t;
   }
   if (lane == 0) {
-    red_z[warp] = static_cast<double>(z) + static_cast<double>(ze);
-    red_s[warp] = static_cast<double>(sv) + static_cast<double>(se);
+    red_z[warp] = make_float2(z, ze);
+    red_s[warp] = make_float2(sv, se);
   }
   __syncthreads();
-  RowOut r{M, I, 0.0, 0.0};
+  RowOut r{M, I, 0.0f, 0.0f};
   if (tid == 0) {
-    for (int w = 0; w < NW; ++w) {
-      r.Z += red_z[w];
-      r.S += red_s[w];
+    // the warps' (value, error) pairs added with TwoSum in fp32 (no fp64: this GPU's fp64 adds
+    // have long latencies, and this runs at the end of every row with no copy in flight)
+    float zh = red_z[0].x, zl = red_z[0].y, sh = red_s[0].x, sl = red_s[0].y;
+#pragma unroll
+    for (int w = 1; w < NW; ++w) {
+      float t, e;
+      two_sum(zh, red_z[w].x, t, e);
+      zl += e + red_z[w].y;
+      zh = t;
+      two_sum(sh, red_s[w].x, t, e);
+      sl += e + red_s[w].y;
+      sh = t;
     }
+    // S / Z with one correction step on the pairs: q = sh / zh, then the residual of
+    // (sh + sl) - q (zh + zl) divided by zh
+    const float q0 = sh / zh;
+    const float res = fmaf(-q0, zh, sh) + (sl - q0 * zl);
+    r.q = q0 + res / zh;
+    r.Z = zh + zl;
   }
   return r;
 }
@@ -211,9 +234,9 @@ __device__ __forceinline__ bool row_write(const RowOut& r, int n, const uint16_t
                                           const int32_t* cur_tok, const float* d_in, const float* d_out, int topk,
                                           float* maxprob, float* entropy, int32_t* argmax, float* score,
                                           uint32_t* counters, float* ws_u = nullptr, float* ws_lnz = nullptr) {
-  const float Zf = static_cast<float>(r.Z);
+  const float Zf = r.Z;
   const float lnZ = logf(Zf);
-  const float H = lnZ - 0.6931471805599453f * static_cast<float>(r.S / r.Z);
+  const float H = lnZ - 0.6931471805599453f * r.q;
   const int y = cur_tok != nullptr ? cur_tok[n] : r.yhat;
   float u = __int_as_float(0x7fc00000);   // a current token outside [0, V) has no probability
   if (y >= 0 && y < V) {
@@ -293,6 +316,21 @@ __device__ __forceinline__ T block_sum(T v, T* scratch) {
   T t = 0;
   for (int w = 0; w < nw; ++w) t += scratch[w];
   return t;
+}
+
+// A finite fp32 score as a 64-bit fixed-point integer on the binade of the segment's largest
+// score (biased exponent emax): s 2^(26 - E), |result| < 2^50. Exact for a score within a factor
+// 2^26 of the largest; a smaller one is truncated toward zero. Sums of up to 4096 of them and
+// their products with counts up to 4096 stay below 2^62, so the mean test n_t s > sum s is an
+// exact integer comparison on these values.
+__device__ __forceinline__ long long fixed_of(float s, uint32_t emax) {
+  const uint32_t bits = __float_as_uint(s);
+  const uint32_t eb = (bits >> 23) & 0xffu;
+  // s = m 2^(eb - 150) (m with its leading bit; a denormal has eb 0 and exponent 1 - 150)
+  const uint32_t m = eb != 0u ? ((bits & 0x7fffffu) | 0x800000u) : (bits & 0x7fffffu);
+  const int shift = static_cast<int>(eb == 0u ? 1u : eb) - static_cast<int>(emax) + 26;
+  const long long mag = shift >= 0 ? (static_cast<long long>(m) << shift) : (shift > -25 ? (m >> -shift) : 0);
+  return (bits >> 31) ? -mag : mag;
 }
 
 // key of row i ordered by value descending, then index ascending; 0 = no row
@@ -465,7 +503,8 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
                                const float* d_in, const float* d_out, float* score) {
   __shared__ int s_ri[32];
   __shared__ int s_nt[32];
-  __shared__ double s_rd[32];
+  __shared__ uint32_t s_em[32];
+  __shared__ long long s_fx[32];
   __shared__ unsigned long long s_top[2][32];
   __shared__ uint64_t s_sel[kRoundsMax];
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5, nw = nt >> 5;
@@ -473,7 +512,7 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
   float* sscore = reinterpret_cast<float*>(keys + sort_n);   // per-row seed score
 
   int n_t = 0;
-  double total = 0.0;
+  uint32_t emax = 0;   // largest biased exponent of the finite scores
   for (int i = tid; i < sort_n; i += nt) {
     uint64_t key = 0;
     if (i < per_seq) {
@@ -487,7 +526,7 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
         if (isfinite(sc)) {
           s = sc;
           ++n_t;
-          total += static_cast<double>(sc);
+          emax = max(emax, (__float_as_uint(sc) >> 23) & 0xffu);
           if ((fl & 1u) == 0 && d.remask_cnt[n] < d.remask_budget) key = rank_key(sc, i);
         }
       }
@@ -498,27 +537,37 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
     keys[i] = key;
   }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    n_t += __shfl_xor_sync(0xffffffffu, n_t, o);
-    total += __shfl_xor_sync(0xffffffffu, total, o);
-  }
+  for (int o = 16; o > 0; o >>= 1) n_t += __shfl_xor_sync(0xffffffffu, n_t, o);
+  emax = __reduce_max_sync(0xffffffffu, emax);
   if (lane == 0) {
     s_nt[warp] = n_t;
-    s_rd[warp] = total;
+    s_em[warp] = emax;
   }
   __syncthreads();
   n_t = 0;
-  total = 0.0;
+  emax = 0;
   for (int w = 0; w < nw; ++w) {
     n_t += s_nt[w];
-    total += s_rd[w];
+    emax = max(emax, s_em[w]);
   }
+  // the sum of the scores, exact in fixed point (fixed_of)
+  long long part = 0;
+  for (int i = tid; i < per_seq; i += nt) {
+    const float s = sscore[i];
+    if (s != -INFINITY) part += fixed_of(s, emax);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+  if (lane == 0) s_fx[warp] = part;
+  __syncthreads();
+  long long total = 0;
+  for (int w = 0; w < nw; ++w) total += s_fx[w];
 
   // adaptive revision rate: n_t pi_t = #{ s_j > mean } = #{ n_t s_j > sum s }
   int above = 0;
   for (int i = tid; i < per_seq; i += nt) {
     const float s = sscore[i];
-    if (s != -INFINITY && static_cast<double>(n_t) * static_cast<double>(s) > total) ++above;
+    if (s != -INFINITY && static_cast<long long>(n_t) * fixed_of(s, emax) > total) ++above;
   }
   above = block_sum(above, s_ri);
   int k = 0;
@@ -646,12 +695,10 @@ __device__ void select_fast(uint64_t* keys, int seg, int per_seq, const DecideAr
       if ((fl & 1u) == 0 && static_cast<int>(rc) < d.remask_budget) key = rank_key(v, tid);
     }
   }
-  // n_t pi_t = #{n_t s_j > sum s} in exact integer arithmetic. Every score becomes a 64-bit
-  // fixed-point integer on the sequence's largest binade: S = s 2^(26 - E) with E the largest
-  // exponent, so |S| < 2^50, exact for every score within a factor 2^26 of the largest (a smaller
-  // one is truncated toward zero; it lies far below the mean, and the sum's error stays below
-  // n_t units, 2^-50 of the largest score). The sum and the products n_t S (|n_t S| < 2^62) are
-  // exact integers; this GPU's fp64 units have long latencies, so no fp64 is used here.
+  // n_t pi_t = #{n_t s_j > sum s} in exact integer arithmetic on the scores' fixed-point values
+  // (fixed_of); a score too small to be exact lies far below the mean, and the sum's error
+  // stays below n_t units, 2^-50 of the largest score. This GPU's fp64 units have long
+  // latencies, so no fp64 is used here.
   const uint32_t sbits = __float_as_uint(sc);
   const uint32_t ebias = valid ? ((sbits >> 23) & 0xffu) : 0u;
   const uint32_t emax_w = __reduce_max_sync(0xffffffffu, ebias);
@@ -667,14 +714,7 @@ __device__ void select_fast(uint64_t* keys, int seg, int per_seq, const DecideAr
     if (eb != 0u) atomicAdd(&s_elig, __popc(eb));
   }
   const int n_t = __syncthreads_count(valid);
-  long long fx = 0;
-  if (valid) {
-    // s = m 2^(ebias - 150) (m with its leading bit; a denormal has ebias 0 and exponent 1 - 150)
-    const uint32_t m = ebias != 0u ? ((sbits & 0x7fffffu) | 0x800000u) : (sbits & 0x7fffffu);
-    const int shift = static_cast<int>(ebias == 0u ? 1u : ebias) - static_cast<int>(s_emax) + 26;
-    const long long mag = shift >= 0 ? (static_cast<long long>(m) << shift) : (shift > -25 ? (m >> -shift) : 0);
-    fx = (sbits >> 31) ? -mag : mag;
-  }
+  const long long fx = valid ? fixed_of(sc, s_emax) : 0;
   long long tot = fx;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
@@ -964,7 +1004,7 @@ __global__ void __launch_bounds__(kThreads, 2) score_kernel(const ScoreParams P)
   extern __shared__ __align__(16) uint64_t keys[];
   __shared__ float red_m[kWarps];
   __shared__ int red_i[kWarps];
-  __shared__ double red_z[kWarps], red_s[kWarps];
+  __shared__ float2 red_z[kWarps], red_s[kWarps];
   __shared__ int s_last;
 
   const int n = blockIdx.x;
@@ -1023,7 +1063,7 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
   __shared__ uint64_t bar_full[kRingStages], bar_empty[kRingStages];
   __shared__ float red_m[kConsumerWarps + 1];
   __shared__ int red_i[kConsumerWarps + 1];
-  __shared__ double red_z[kConsumerWarps + 1], red_s[kConsumerWarps + 1];
+  __shared__ float2 red_z[kConsumerWarps + 1], red_s[kConsumerWarps + 1];
   __shared__ int s_last, s_abort;
 
   const int n = blockIdx.x;
