@@ -13,9 +13,10 @@
 // Then c = 1/Z, H = ln Z - ln(2) S / Z, u = ln Z - (x_y - m).
 //
 // Top-k (Section 5.3): the last CTA to finish a segment (sequence) - found
-// with a self-resetting atomicInc counter per segment - sorts the segment's
-// eligible rows by (score descending, index ascending) with a bitonic sort of
-// 64-bit keys in shared memory and writes the first k.
+// with a self-resetting counter per segment, incremented with acquire-release
+// semantics - takes the segment's k best eligible rows by (score descending,
+// index ascending) on 64-bit keys: by rank when every row has its own thread,
+// else by warp sorts and merges (k <= 32) or a bitonic sort in shared memory.
 //
 // Decision step (cover_score_decide_fwd, Sections 5.2, 3 and 5.3): the row
 // pass keeps u of the current token and ln Z (= u of the greedy token) in a
@@ -54,11 +55,13 @@ constexpr int kChunkBytes = kChunkElems * 2;
 constexpr int kRingStages = 3;
 constexpr int kVecPerThread = kChunkElems / 8 / (kConsumerWarps * 32);   // 4
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr int kRoundsMax = 32;             // decision step: selections up to this size by rounds
+constexpr int kRoundsMax = 32;             // selections up to this size by warp sorts (top_warps)
 
 struct RowAcc {
   float m;     // running maximum logit of this thread's elements
-  int mi;      // first index where it occurs
+  int mi;      // where m was first reached: the element's index (mu == 0), else the first index of
+               // the batch that held it, mu vectors of 8 values a kernel-constant stride apart
+  int mu;
   float mref;  // m * log2(e), the exponent reference
   float z, zc; // Kahan sum of 2^t and its compensation
   float s, sc; // Kahan sum of t 2^t and its compensation
@@ -72,7 +75,7 @@ __device__ __forceinline__ void kahan_add(float& sum, float& c, float x) {
 }
 
 // Move the exponent reference to a larger maximum new_m.
-__device__ __forceinline__ void raise_max(RowAcc& a, float new_m, int new_i) {
+__device__ __forceinline__ void raise_max(RowAcc& a, float new_m, int new_i, int new_u) {
   const float new_ref = new_m * kLog2e;
   if (a.m != -INFINITY) {
     const float d = a.mref - new_ref;  // <= 0
@@ -86,6 +89,7 @@ __device__ __forceinline__ void raise_max(RowAcc& a, float new_m, int new_i) {
   a.sc = 0.0f;
   a.m = new_m;
   a.mi = new_i;
+  a.mu = new_u;
   a.mref = new_ref;
 }
 
@@ -100,7 +104,7 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
 __device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
 
 __device__ __forceinline__ void acc_scalar(RowAcc& a, float x, int idx) {
-  if (x > a.m) raise_max(a, x, idx);
+  if (x > a.m) raise_max(a, x, idx, 0);
   const float t = fmaf(x, kLog2e, -a.mref);
   const float e = ex2_approx(t);
   kahan_add(a.z, a.zc, e);
@@ -142,37 +146,51 @@ __device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
   e = (a - (s - bb)) + (b - bb);
 }
 
-template <int NW>
-__device__ __forceinline__ RowOut row_reduce(const RowAcc& a, float* red_m, int* red_i, float2* red_z,
-                                             float2* red_s) {
+// A thread's recorded batch is re-read from the row in global memory, in up to four vectors
+// kStride elements apart; the loads are issued by the threads that hold their warp's maximum
+// before the block-wide maximum is known, so their latency overlaps the reduction.
+constexpr int kMaxBatch = 4;
+static_assert(kVecPerThread <= kMaxBatch && kUnroll <= kMaxBatch, "batches hold at most four vectors");
+
+template <int kStride>
+__device__ __forceinline__ void load_batch(const RowAcc& a, const uint16_t* row, uint4 (&w)[kMaxBatch]) {
+#pragma unroll
+  for (int u = 0; u < kMaxBatch; ++u)
+    if (u < a.mu) w[u] = ld_stream(reinterpret_cast<const uint4*>(row + a.mi + u * kStride));
+}
+
+// First index of the value M in the thread's recorded batch w.
+template <int kStride>
+__device__ __forceinline__ int first_index_of(const RowAcc& a, float M, const uint4 (&w)[kMaxBatch]) {
+  if (a.mu == 0) return a.mi;
+  int idx = 0x7fffffff;
+#pragma unroll
+  for (int u = kMaxBatch - 1; u >= 0; --u) {
+    if (u >= a.mu) continue;
+    float x[8];
+    unpack8(w[u], x);
+#pragma unroll
+    for (int k = 7; k >= 0; --k)
+      if (x[k] == M) idx = a.mi + u * kStride + k;
+  }
+  return idx;
+}
+
+template <int NW, int kStride>
+__device__ __forceinline__ RowOut row_reduce(const RowAcc& a, const uint16_t* row, float* red_m, int* red_i,
+                                             float2* red_z, float2* red_s) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   float m = a.m;
-  int mi = a.mi;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
-    const int i2 = __shfl_xor_sync(0xffffffffu, mi, o);
-    if (m2 > m || (m2 == m && i2 < mi)) {
-      m = m2;
-      mi = i2;
-    }
-  }
-  if (lane == 0) {
-    red_m[warp] = m;
-    red_i[warp] = mi;
-  }
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  const bool cand = a.m == m && m != -INFINITY;   // may hold the row maximum
+  uint4 w[kMaxBatch];
+  if (cand) load_batch<kStride>(a, row, w);
+  if (lane == 0) red_m[warp] = m;
   __syncthreads();
   float M = red_m[0];
-  int I = red_i[0];
 #pragma unroll
-  for (int w = 1; w < NW; ++w) {
-    const float m2 = red_m[w];
-    const int i2 = red_i[w];
-    if (m2 > M || (m2 == M && i2 < I)) {
-      M = m2;
-      I = i2;
-    }
-  }
+  for (int i = 1; i < NW; ++i) M = fmaxf(M, red_m[i]);
   const float Mref = M * kLog2e;
   // partials re-referenced to the row maximum, summed across the warp in fp32
   // with error-free TwoSum pairs (value, rounding error), then across the warps
@@ -198,13 +216,20 @@ __device__ __forceinline__ RowOut row_reduce(const RowAcc& a, float* red_m, int*
     se += se2 + ((sv - (t - bb)) + (s2 - bb));
     sv = t;
   }
+  // the threads holding the row maximum find its first index in their recorded batches
+  const int mi = __reduce_min_sync(0xffffffffu, cand && a.m == M ? first_index_of<kStride>(a, M, w) : 0x7fffffff);
   if (lane == 0) {
+    red_i[warp] = mi;
     red_z[warp] = make_float2(z, ze);
     red_s[warp] = make_float2(sv, se);
   }
   __syncthreads();
-  RowOut r{M, I, 0.0f, 0.0f};
+  RowOut r{M, 0x7fffffff, 0.0f, 0.0f};
   if (tid == 0) {
+    int I = red_i[0];
+#pragma unroll
+    for (int w = 1; w < NW; ++w) I = min(I, red_i[w]);
+    r.yhat = I;
     // the warps' (value, error) pairs added with TwoSum in fp32 (no fp64: this GPU's fp64 adds
     // have long latencies, and this runs at the end of every row with no copy in flight)
     float zh = red_z[0].x, zl = red_z[0].y, sh = red_s[0].x, sl = red_s[0].y;
@@ -256,9 +281,14 @@ __device__ __forceinline__ bool row_write(const RowOut& r, int n, const uint16_t
     score[n] = u * (1.0f + din) / (1.0f + dout);
     if (topk <= 0) return false;
   }
-  __threadfence();
+  // The counter increment is a release (thread 0 wrote all of the row's results above) and an
+  // acquire: the segment's last CTA, after its block barrier, reads the results of the others.
   const unsigned seg = static_cast<unsigned>(n / per_seq);
-  const unsigned old = atomicInc(counters + seg, static_cast<unsigned>(per_seq - 1));
+  unsigned old;
+  asm volatile("atom.acq_rel.gpu.global.inc.u32 %0, [%1], %2;"
+               : "=r"(old)
+               : "l"(counters + seg), "r"(static_cast<unsigned>(per_seq - 1))
+               : "memory");
   return old == static_cast<unsigned>(per_seq - 1);
 }
 
@@ -341,36 +371,104 @@ __device__ __forceinline__ int rank_key_row(uint64_t key) {
   return static_cast<int>(0xffffffffu - static_cast<uint32_t>(key));
 }
 
-// The k largest of the n keys in shared memory (keys are distinct, 0 = none),
-// in descending order, by k rounds of a CTA-wide maximum below the previous
-// round's: one barrier per round, the keys untouched. out[t] gets round t's
-// key (0 once the nonzero keys run out). All threads call it with the same k.
-__device__ __forceinline__ void top_rounds(const uint64_t* keys, int n, int k, uint64_t* out,
-                                           unsigned long long (*scratch)[32]) {
-  const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5, nw = nt >> 5;
-  uint64_t prev = ~0ull;
-  for (int t = 0; t < k; ++t) {
-    uint64_t m = 0;
-    for (int i = tid; i < n; i += nt) {
-      const uint64_t x = keys[i];
-      if (x < prev && x > m) m = x;
-    }
+// Descending bitonic sorts of G independent sets of 32 keys across the warp (key[g]: lane t's
+// key of set g), by shuffles; the G sets go through the network together.
+template <int G>
+__device__ __forceinline__ void warp_sort_desc(uint64_t (&key)[G], int lane) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const uint64_t y = __shfl_xor_sync(0xffffffffu, m, o);
-      m = y > m ? y : m;
-    }
-    if (lane == 0) scratch[t & 1][warp] = m;
-    __syncthreads();
-    m = 0;
-    for (int w = 0; w < nw; ++w) m = scratch[t & 1][w] > m ? scratch[t & 1][w] : m;
-    if (tid == 0) out[t] = m;
-    prev = m;
-    if (m == 0) {
-      for (int r = t + 1 + tid; r < k; r += nt) out[r] = 0;
-      break;
+  for (int size = 2; size <= 32; size <<= 1) {
+    const bool desc = (lane & size) == 0;
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const bool take_max = ((lane & stride) == 0) == desc;
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        const uint64_t other = __shfl_xor_sync(0xffffffffu, key[g], stride);
+        key[g] = take_max ? (key[g] > other ? key[g] : other) : (key[g] < other ? key[g] : other);
+      }
     }
   }
+}
+__device__ __forceinline__ uint64_t warp_sort_desc(uint64_t key, int lane) {
+  uint64_t k1[1] = {key};
+  warp_sort_desc<1>(k1, lane);
+  return k1[0];
+}
+
+// a[g] becomes the 32 largest of the descending lists a[g] and b[g] (lane t holds the t-th of
+// each), descending: the larger of a[t] and b[31 - t] is a bitonic sequence holding them, which
+// the half-cleaners of strides 16 .. 1 put in order. The G merges go through together.
+template <int G>
+__device__ __forceinline__ void warp_merge_desc(uint64_t (&a)[G], const uint64_t (&b)[G], int lane) {
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    const uint64_t br = __shfl_sync(0xffffffffu, b[g], 31 - lane);
+    a[g] = a[g] > br ? a[g] : br;
+  }
+#pragma unroll
+  for (int stride = 16; stride > 0; stride >>= 1) {
+    const bool take_max = (lane & stride) == 0;
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const uint64_t other = __shfl_xor_sync(0xffffffffu, a[g], stride);
+      a[g] = take_max ? (a[g] > other ? a[g] : other) : (a[g] < other ? a[g] : other);
+    }
+  }
+}
+
+// Number of entries of the descending list l[0 .. 32) larger than x (x not in the list).
+__device__ __forceinline__ int count_above(const uint64_t* l, uint64_t x) {
+  int c = 0;
+#pragma unroll
+  for (int step = 32; step > 0; step >>= 1)
+    if (c + step <= 32 && l[c + step - 1] > x) c += step;
+  return c;
+}
+
+// The k largest (k <= 32) of the n keys in shared memory (distinct, 0 = none), in descending
+// order: out[t] gets the t-th (0 once the nonzero keys run out). Each warp keeps the 32 largest
+// keys it has read in registers (lane t: the t-th). It reads four sets of 32 keys at a time
+// (every (warps)-th set of the array), sorts them together, merges them pairwise and folds the
+// result into its list, skipping the work when no key passes the list's k-th. A key can be
+// among the k largest only if it is among its warp's, so the warps' lists decide the result:
+// a listed key's rank is its position in its own list plus the number of larger keys in each
+// other list (a binary search, the lists being sorted), exact below k. The lists are staged in
+// keys[0 .. 32 * warps), which n >= blockDim.x guarantees; the keys are not read afterwards.
+// All threads call it with the same k.
+__device__ __forceinline__ void top_warps(uint64_t* keys, int n, int k, uint64_t* out) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+  if (k <= 0) return;
+  constexpr int kSets = 4;
+  uint64_t top[1] = {0};
+  for (int j0 = warp * 32 + lane; j0 - lane < n; j0 += kSets * nw * 32) {
+    uint64_t b[kSets];
+#pragma unroll
+    for (int g = 0; g < kSets; ++g) {
+      const int j = j0 + g * nw * 32;
+      b[g] = j < n ? keys[j] : 0;
+    }
+    const uint64_t kth = __shfl_sync(0xffffffffu, top[0], k - 1);
+    if (!__any_sync(0xffffffffu, b[0] > kth || b[1] > kth || b[2] > kth || b[3] > kth)) continue;
+    warp_sort_desc<kSets>(b, lane);
+    uint64_t p[2] = {b[0], b[2]};
+    const uint64_t q[2] = {b[1], b[3]};
+    warp_merge_desc<2>(p, q, lane);
+    const uint64_t p1[1] = {p[1]};
+    uint64_t p0[1] = {p[0]};
+    warp_merge_desc<1>(p0, p1, lane);
+    warp_merge_desc<1>(top, p0, lane);
+  }
+  __syncthreads();   // every warp is done reading the keys
+  keys[warp * 32 + lane] = lane < k ? top[0] : 0;
+  const int published = __syncthreads_count(lane < k && top[0] != 0);
+  if (lane < k && top[0] != 0) {
+    int r = lane;
+#pragma unroll 4
+    for (int w = 0; w < nw; ++w)
+      if (w != warp) r += count_above(keys + w * 32, top[0]);
+    if (r < k) out[r] = top[0];
+  }
+  for (int t = min(published, k) + tid; t < k; t += blockDim.x) out[t] = 0;
   __syncthreads();
 }
 
@@ -384,9 +482,7 @@ __device__ void segment_update(uint64_t* keys, int seg, int per_seq, int sort_n,
   __shared__ unsigned long long s_fallback;
   __shared__ int s_ri[32];
   __shared__ int s_cnt[3][32];
-  __shared__ unsigned long long s_top[2][32];
   __shared__ uint64_t s_sel[kRoundsMax];
-  __threadfence();
   const DecideArgs& d = P.dec;
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5, nw = nt >> 5;
   const int base = seg * per_seq;
@@ -423,7 +519,7 @@ __device__ void segment_update(uint64_t* keys, int seg, int per_seq, int sort_n,
     }
     __syncthreads();
     if (n_drafted <= kRoundsMax)
-      top_rounds(keys, sort_n, n_drafted, s_sel, s_top);
+      top_warps(keys, sort_n, n_drafted, s_sel);
     else
       bitonic_sort_desc(keys, sort_n);
   }
@@ -505,7 +601,6 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
   __shared__ int s_nt[32];
   __shared__ uint32_t s_em[32];
   __shared__ long long s_fx[32];
-  __shared__ unsigned long long s_top[2][32];
   __shared__ uint64_t s_sel[kRoundsMax];
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5, nw = nt >> 5;
   const int base = seg * per_seq;
@@ -577,7 +672,7 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
   // the k best eligible rows (keys written above)
   const uint64_t* best = keys;
   if (k > 0 && k <= kRoundsMax) {
-    top_rounds(keys, sort_n, k, s_sel, s_top);
+    top_warps(keys, sort_n, k, s_sel);
     best = s_sel;
   } else if (k > 0) {
     bitonic_sort_desc(keys, sort_n);
@@ -613,7 +708,7 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
 // other candidates' keys in shared memory: its rank is the number of larger
 // keys, so the row of rank r < k is the (r+1)-th best and fills slot r. Keys
 // embed the row index, so they are distinct and the result is the general
-// path's (the sort or the rounds of maxima) exactly.
+// path's (the sort or the warp sorts) exactly.
 // ---------------------------------------------------------------------------
 
 // Rank of x among keys[0 .. n) (16-byte aligned): the number of larger keys, counted only while
@@ -636,20 +731,6 @@ __device__ __forceinline__ int rank_below(const uint64_t* keys, int n, uint64_t 
   return r;
 }
 
-// Descending bitonic sort of a warp's 32 keys, one per lane, by shuffles.
-__device__ __forceinline__ uint64_t warp_sort_desc(uint64_t key, int lane) {
-#pragma unroll
-  for (int size = 2; size <= 32; size <<= 1) {
-    const bool desc = (lane & size) == 0;
-#pragma unroll
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      const uint64_t other = __shfl_xor_sync(0xffffffffu, key, stride);
-      const bool take_max = ((lane & stride) == 0) == desc;
-      key = take_max ? (key > other ? key : other) : (key < other ? key : other);
-    }
-  }
-  return key;
-}
 
 // The k largest (k <= 32) of the CTA's keys, one per thread (distinct, 0 = none). Each warp sorts
 // its keys and publishes its k largest in cand[warp * k ..]; a key can be among the CTA's k
@@ -770,7 +851,6 @@ __device__ void decide_fast(uint64_t* keys, int seg, int per_seq, const ScorePar
   __shared__ unsigned long long s_fallback;
   __shared__ int s_cnt[3];
   __shared__ uint8_t s_draft[512];   // blockDim <= 512
-  __threadfence();
   const DecideArgs& d = P.dec;
   const int tid = threadIdx.x, lane = tid & 31;
   const bool in = tid < per_seq;
@@ -896,16 +976,16 @@ __device__ void segment_decide(uint64_t* keys, int seg, int per_seq, int sort_n,
 __device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_seq, int sort_n, int topk,
                                              const float* score, const uint8_t* eligible, int32_t* topk_idx,
                                              float* topk_score) {
-  __threadfence();
   const int tid = threadIdx.x, nt = blockDim.x;
   const int base = seg * per_seq;
   if (per_seq <= nt) {
     // one row per thread: rank every eligible row against the others (see decide_fast)
     uint64_t key = 0;
     float sc = 0.0f;
-    if (tid < per_seq && (eligible == nullptr || eligible[base + tid] != 0)) {
+    if (tid < per_seq) {
+      // both loads issued together: the score is read whether or not the row is eligible
       sc = __ldcg(score + base + tid);
-      key = rank_key(sc, tid);
+      if (eligible == nullptr || eligible[base + tid] != 0) key = rank_key(sc, tid);
     }
     if (tid < per_seq) keys[tid] = key;
     const int n_elig = __syncthreads_count(key != 0);
@@ -922,21 +1002,31 @@ __device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_se
     }
     return;
   }
-  for (int i = tid; i < sort_n; i += nt) {
-    uint64_t key = 0;
-    if (i < per_seq && (eligible == nullptr || eligible[base + i] != 0)) {
-      const float sc = __ldcg(score + base + i);
-      key = (static_cast<uint64_t>(order_key(sc)) << 32) | (0xffffffffu - static_cast<uint32_t>(i));
+  // the scores and flags of kLoads rows per thread are loaded before any key is stored, so the
+  // loads of a thread overlap instead of waiting one after the other
+  constexpr int kLoads = 4;
+  for (int i0 = tid; i0 < sort_n; i0 += kLoads * nt) {
+    float sc[kLoads];
+    bool el[kLoads];
+#pragma unroll
+    for (int u = 0; u < kLoads; ++u) {
+      const int i = i0 + u * nt;
+      const bool in = i < per_seq;
+      sc[u] = in ? __ldcg(score + base + i) : 0.0f;
+      el[u] = in && (eligible == nullptr || eligible[base + i] != 0);
     }
-    keys[i] = key;
+#pragma unroll
+    for (int u = 0; u < kLoads; ++u) {
+      const int i = i0 + u * nt;
+      if (i < sort_n) keys[i] = el[u] ? rank_key(sc[u], i) : 0;
+    }
   }
   __syncthreads();
-  // a short list by rounds of maxima (one barrier each), a long one by sorting
-  __shared__ unsigned long long s_top[2][32];
+  // a short list by warp sorts and merges, a long one by sorting
   __shared__ uint64_t s_sel[kRoundsMax];
   const uint64_t* best = keys;
   if (topk <= kRoundsMax) {
-    top_rounds(keys, sort_n, topk, s_sel, s_top);
+    top_warps(keys, sort_n, topk, s_sel);
     best = s_sel;
   } else {
     bitonic_sort_desc(keys, sort_n);
@@ -952,11 +1042,12 @@ __device__ __forceinline__ void segment_topk(uint64_t* keys, int seg, int per_se
   }
 }
 
-// Accumulate U vectors of 8 values; the first index of vector u is i0 + u * istride.
+// Accumulate U vectors of 8 values; the first index of vector u is i0 + u * istride, istride
+// being the kernel's constant batch stride when U > 1.
 // Per pair of values: one packed FMA for t, two ex2, one packed add into Z and
 // one packed FMA into S; two independent accumulator chains.
 template <int U>
-__device__ __forceinline__ void acc_batch(RowAcc& a, const uint4 (&w)[U], int i0, int istride) {
+__device__ __forceinline__ void acc_batch(RowAcc& a, const uint4 (&w)[U], int i0) {
   float x[U][8];
   float bmax = -INFINITY;
 #pragma unroll
@@ -965,15 +1056,9 @@ __device__ __forceinline__ void acc_batch(RowAcc& a, const uint4 (&w)[U], int i0
 #pragma unroll
     for (int k = 0; k < 8; k += 2) bmax = fmax3(bmax, x[u][k], x[u][k + 1]);
   }
-  if (bmax > a.m) {
-    int idx = 0x7fffffff;
-#pragma unroll
-    for (int u = U - 1; u >= 0; --u)
-#pragma unroll
-      for (int k = 7; k >= 0; --k)
-        if (x[u][k] == bmax) idx = i0 + u * istride + k;
-    raise_max(a, bmax, idx);
-  }
+  // the batch is recorded, not searched: only the row maximum's first index is needed, and
+  // row_reduce finds it in the recorded batches of the threads that hold that maximum
+  if (bmax > a.m) raise_max(a, bmax, i0, U);
   const uint64_t c2 = f2_pack(kLog2e, kLog2e);
   const uint64_t nm2 = f2_pack(-a.mref, -a.mref);
   uint64_t z[2] = {0, 0}, sacc[2] = {0, 0};
@@ -1012,7 +1097,7 @@ __global__ void __launch_bounds__(kThreads, 2) score_kernel(const ScoreParams P)
   const int V = P.V;
   const size_t row_off = static_cast<size_t>(n) * V;
   const uint16_t* row = P.logits + row_off;
-  RowAcc a{-INFINITY, 0x7fffffff, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+  RowAcc a{-INFINITY, 0x7fffffff, 0, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
 
   // elements before the first 16-byte boundary of the row
   const int head = min(static_cast<int>((8 - (row_off & 7)) & 7), V);
@@ -1025,15 +1110,15 @@ __global__ void __launch_bounds__(kThreads, 2) score_kernel(const ScoreParams P)
     uint4 w[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) w[u] = ld_stream(vrow + v + u * kThreads);
-    acc_batch<kUnroll>(a, w, head + v * 8, kThreads * 8);
+    acc_batch<kUnroll>(a, w, head + v * 8);
   }
   for (; v < nvec; v += kThreads) {
     uint4 w[1] = {ld_stream(vrow + v)};
-    acc_batch<1>(a, w, head + v * 8, 0);
+    acc_batch<1>(a, w, head + v * 8);
   }
   if (tail0 + tid < V) acc_scalar(a, bf16_to_f32(row[tail0 + tid]), tail0 + tid);
 
-  const RowOut r = row_reduce<kWarps>(a, red_m, red_i, red_z, red_s);
+  const RowOut r = row_reduce<kWarps, kThreads * 8>(a, row, red_m, red_i, red_z, red_s);
   if (tid == 0)
     s_last = row_write(r, n, row, V, P.per_seq, P.decide ? P.dec.tok : P.cur_tok, P.d_in, P.d_out, P.topk,
                        P.maxprob, P.entropy, P.argmax, P.score, P.counters, P.decide ? P.dec.ws_u : nullptr,
@@ -1091,7 +1176,7 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
   }
   __syncthreads();
 
-  RowAcc a{-INFINITY, 0x7fffffff, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+  RowAcc a{-INFINITY, 0x7fffffff, 0, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
   if (warp == kConsumerWarps) {
     // producer: one lane streams the row chunk by chunk
     if (lane == 0) {
@@ -1129,11 +1214,11 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
         uint4 w[kVecPerThread];
 #pragma unroll
         for (int u = 0; u < kVecPerThread; ++u) w[u] = src[tid + u * kStride];
-        acc_batch<kVecPerThread>(a, w, c * kChunkElems + tid * 8, kStride * 8);
+        acc_batch<kVecPerThread>(a, w, c * kChunkElems + tid * 8);
       } else {
         for (int v = tid; v < nv; v += kStride) {
           uint4 w[1] = {src[v]};
-          acc_batch<1>(a, w, c * kChunkElems + v * 8, 0);
+          acc_batch<1>(a, w, c * kChunkElems + v * 8);
         }
       }
       __syncwarp();
@@ -1146,7 +1231,7 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
       mbar_wait(&bar_full[c % kRingStages], (c / kRingStages) & 1, nullptr, 1000000ull);
   }
 
-  const RowOut r = row_reduce<kConsumerWarps + 1>(a, red_m, red_i, red_z, red_s);
+  const RowOut r = row_reduce<kConsumerWarps + 1, kConsumerWarps * 32 * 8>(a, row, red_m, red_i, red_z, red_s);
   if (tid == 0)
     s_last = row_write(r, n, row, V, P.per_seq, P.decide ? P.dec.tok : P.cur_tok, P.d_in, P.d_out, P.topk,
                        P.maxprob, P.entropy, P.argmax, P.score, P.counters, P.decide ? P.dec.ws_u : nullptr,

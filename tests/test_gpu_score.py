@@ -61,6 +61,18 @@ def test_score_side_inputs_and_eligibility():
     check(inp, run_score(inp))
 
 
+@pytest.mark.parametrize("per,k", [(1000, 32), (300, 20)])
+def test_score_topk_fewer_eligible_than_k(per, k):
+    """General path with fewer eligible rows than k: the list ends in -1 / -inf."""
+    inp = W.make_score_inputs(2 * per, 300, 2, k, seed=per, eligible_frac=0.012)
+    r = run_score(inp)
+    check(inp, r)
+    n_elig = inp.eligible.reshape(2, per).sum(axis=1)
+    assert (n_elig < k).all()
+    for g in range(2):
+        assert (r["topk_idx"][g, n_elig[g]:] == -1).all() and (r["topk_idx"][g, :n_elig[g]] >= 0).all()
+
+
 def test_score_no_eligible_rows():
     inp = W.make_score_inputs(32, 512, 2, 4, seed=8, eligible_frac=0.0)
     r = run_score(inp)
@@ -77,6 +89,35 @@ def test_score_ties_and_uniform_rows():
     inp.logits = x
     r = run_score(inp)
     assert r["argmax"][0] == 0 and r["argmax"][1] == 17
+    check(inp, r)
+
+
+@pytest.mark.parametrize("V", [40000, 40001])   # bulk-copy kernel (V % 8 == 0), register-load kernel
+def test_score_argmax_ties_across_batches(V):
+    """The first index of the row maximum when it occurs several times: in different chunks, in one
+    thread's batch (different vectors), in one thread's batches of different chunks, at the row's
+    first and last element, and as -0.0 before +0.0."""
+    placed = [
+        [39999, 12345, 8192 + 3, 20000],       # several chunks: 8195
+        [2 * 2048 + 5 * 8 + 3, 5 * 8 + 6],     # one thread, one batch, vectors 2 and 0: 46
+        [3 * 8192 + 7 * 8 + 1, 8192 + 7 * 8 + 2],
+        [0, V - 1],
+        [V - 1],
+        [8 * 4096 + 11, 4096 + 3, 2 * 4096 + 3],
+    ]
+    inp = W.make_score_inputs(len(placed) + 1, V, 1, 3, seed=V)
+    x = inp.logits.copy()
+    for r, pos in enumerate(placed):
+        x[r, pos] = W.f32_to_bf16_bits(np.full(len(pos), 9.5, np.float32))
+    zr = len(placed)
+    x[zr, :] = W.f32_to_bf16_bits(np.full(V, -2.0, np.float32))
+    x[zr, 30000] = np.uint16(0x8000)   # -0.0
+    x[zr, 31000] = np.uint16(0x0000)   # +0.0
+    x[zr, 500] = np.uint16(0x8000)
+    inp.logits = x
+    r = run_score(inp)
+    expect = [min(p) for p in placed] + [500]
+    assert r["argmax"].tolist() == expect
     check(inp, r)
 
 
@@ -102,10 +143,12 @@ def test_score_named_workloads_full(name):
 
 @pytest.mark.parametrize("per,V,k", [
     (288, 1000, 40),    # one row per thread of the bulk-copy kernel: selection by rank
-    (289, 1000, 20),    # the general path, a short list: rounds of maxima
+    (289, 1000, 20),    # the general path, a short list: warp sorts and merges
     (289, 1000, 40),    # the general path, a long list: the bitonic sort
     (512, 1001, 33),    # the register-load kernel (512 threads): selection by rank
-    (513, 1001, 32),    # and one row past it: rounds of maxima
+    (513, 1001, 32),    # and one row past it: warp sorts and merges
+    (4096, 136, 32),    # the largest segment, k = 32
+    (777, 200, 1),      # k = 1
 ])
 def test_score_topk_on_both_sides_of_the_fast_path(per, V, k):
     inp = W.make_score_inputs(2 * per, V, 2, k, seed=per + k, spike_frac=0.1, eligible_frac=0.8)
