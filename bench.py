@@ -428,14 +428,39 @@ def run_ours(args):
     return result if rank == 0 else None
 
 
-def busy_ahead(torch):
-    """Occupy the device for ~0.1 ms before a timed call.
+def busy_ahead(torch, launches=1):
+    """Occupy the device for ~0.1 ms (plus ~30 us per further launch) before timed calls.
 
-    The call's host-side work (argument checks, the ctypes call) then overlaps
-    this spin, so the events around the call measure device work only rather
-    than also the time the device waited for the launch.
+    The calls' host-side work (argument checks, the ctypes call) then overlaps
+    this spin, so the events around the calls measure device work only rather
+    than also the time the device waited for the launches.
     """
-    torch.cuda._sleep(200_000)
+    torch.cuda._sleep(200_000 + 60_000 * (launches - 1))
+
+
+def time_launches(torch, fn, iters=20, block_us=250.0):
+    """Median device time of one call of `fn` (which must leave its inputs as it found them, or
+    change nothing its work depends on), and the block size used.
+
+    Each of the `iters` samples times a block of R back-to-back calls behind a device spin and
+    divides by R; R is chosen so that a block lasts about `block_us`, because the CUDA event
+    timestamps advance in steps of ~1 us, a few percent of a short launch.
+    """
+    stream = torch.cuda.current_stream()
+
+    def sample(R):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        busy_ahead(torch, R)
+        a.record(stream)
+        for _ in range(R):
+            fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / R
+
+    first = statistics.median(sample(1) for _ in range(3))
+    R = max(1, min(16, round(block_us / (first * 1e3))))
+    return statistics.median(sample(R) for _ in range(iters)), R
 
 
 def score_gbs(api, torch, si, iters=20):
@@ -443,18 +468,9 @@ def score_gbs(api, torch, si, iters=20):
     logits = bf16_dev(si.logits, torch)
     wsp = api.score_workspace(si.n_seq)
     out = api.cover_score_fwd(logits, si.n_seq, si.topk, workspace=wsp)
-    stream = torch.cuda.current_stream()
-    ts = []
-    for _ in range(iters):
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        busy_ahead(torch)
-        a.record(stream)
-        api.cover_score_fwd(logits, si.n_seq, si.topk, workspace=wsp, out=out)
-        b.record(stream)
-        torch.cuda.synchronize()
-        ts.append(a.elapsed_time(b))
+    t, _ = time_launches(torch, lambda: api.cover_score_fwd(logits, si.n_seq, si.topk, workspace=wsp, out=out), iters)
     nbytes = si.N * si.V * 2 + si.N * 20 + si.n_seq * si.topk * 8
-    return round(nbytes / (statistics.median(ts) * 1e-3) / 1e9, 1)
+    return round(nbytes / (t * 1e-3) / 1e9, 1)
 
 
 def decide_timing(api, torch, wl, iters=20):
@@ -554,6 +570,13 @@ def mass_timing(api, torch, wl, q, kc, km, seeds, lse, iters=20):
             torch.cuda.synchronize()
             ts[k].append(a.elapsed_time(b))
     med = {k: statistics.median(v) for k, v in ts.items()}
+    # the mass pass only reads the state: also timed over blocks of back-to-back calls, on the
+    # state the update phase leaves
+    tok.copy_(tok0)
+    flags.copy_(flags0)
+    rc.copy_(rc0)
+    phases["update"]()
+    med["mass"], _ = time_launches(torch, phases["mass"], iters)
     # tensor work of the mass pass: Q K'^T of the response block, 2 * per^2 * D per head
     flops = 2.0 * wl.B * wl.Hq * per * per * wl.D
     return {"response_rows": per, "ms_update": round(med["update"], 4), "ms_mass": round(med["mass"], 4),
@@ -577,24 +600,16 @@ def prefix_timing(api, torch, q, kc, vc, km, vm, seeds, Lq, peak, hbm_gbs, iters
     qw = q[:, :, q0:].contiguous()
     out = torch.empty_like(qw)
     lse = torch.empty((B, Hq, Lq), dtype=torch.float32, device=q.device)
-    stream = torch.cuda.current_stream()
     for _ in range(3):
         api.cover_attn_fwd_prefix(qw, kc, vc, km, vm, seeds, q0=q0, out=out, lse=lse)
-    ts = []
-    for _ in range(iters):
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        busy_ahead(torch)
-        a.record(stream)
-        api.cover_attn_fwd_prefix(qw, kc, vc, km, vm, seeds, q0=q0, out=out, lse=lse)
-        b.record(stream)
-        torch.cuda.synchronize()
-        ts.append(a.elapsed_time(b))
-    t = statistics.median(ts)
+    t, R = time_launches(torch, lambda: api.cover_attn_fwd_prefix(qw, kc, vc, km, vm, seeds, q0=q0, out=out,
+                                                                  lse=lse), iters)
     flops = 4.0 * B * Hq * Lq * L * D
     nbytes = 2 * (2 * B * Hq * Lq * D) + 2 * (2 * B * Hkv * L * D) + 2 * (2 * Hkv * s_in * D) + 4 * B * S \
         + 4 * B * Hq * Lq
     gbs = nbytes / (t * 1e-3) / 1e9
-    return {"Lq": Lq, "Lk": L, "q0": q0, "ms": round(t, 4), "tflops": round(flops / (t * 1e-3) / 1e12, 2),
+    return {"Lq": Lq, "Lk": L, "q0": q0, "ms": round(t, 4), "launches_per_sample": R,
+            "tflops": round(flops / (t * 1e-3) / 1e12, 2),
             "frac_of_peak": round(flops / (t * 1e-3) / 1e12 / peak, 4), "algorithmic_bytes": nbytes,
             "gbs": round(gbs, 1), "frac_of_measured_hbm": round(gbs / hbm_gbs, 4)}
 
@@ -602,31 +617,27 @@ def prefix_timing(api, torch, q, kc, vc, km, vm, seeds, Lq, peak, hbm_gbs, iters
 def kv_timing(api, torch, k, v, seeds, iters=20):
     """Per-layer seed K/V cache traffic: gather at selection, override swap at the next step.
 
-    Times each call alone (median of `iters`); GB/s counts the bytes each call
-    moves (gather: read the seed rows, write the cache; override: read and
-    write both the seed rows and the cache rows, for k and v).
+    Median time of one call (time_launches); GB/s counts the bytes each call moves (gather: read
+    the seed rows, write the cache; override: read and write both the seed rows and the cache
+    rows, for k and v).
     """
     B, Hkv, L, D = k.shape
     S = seeds.shape[1]
-    stream = torch.cuda.current_stream()
     kc, vc = api.cover_seed_kv_gather(k, v, seeds)
+    n_swaps = [0]
 
-    def timed(fn, warm=4):
-        for _ in range(warm):
-            fn()
-        ts = []
-        for _ in range(iters):
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            busy_ahead(torch)
-            a.record(stream)
-            fn()
-            b.record(stream)
-            torch.cuda.synchronize()
-            ts.append(a.elapsed_time(b))
-        return statistics.median(ts)
+    def swap():
+        api.cover_seed_kv_override(k, v, seeds, kc, vc)
+        n_swaps[0] += 1
 
-    t_g = timed(lambda: api.cover_seed_kv_gather(k, v, seeds, k_cache=kc, v_cache=vc))
-    t_o = timed(lambda: api.cover_seed_kv_override(k, v, seeds, kc, vc))   # 24 swaps: k, v end as they began
+    for _ in range(4):
+        api.cover_seed_kv_gather(k, v, seeds, k_cache=kc, v_cache=vc)
+        swap()
+    t_g, _ = time_launches(torch, lambda: api.cover_seed_kv_gather(k, v, seeds, k_cache=kc, v_cache=vc), iters)
+    t_o, _ = time_launches(torch, swap, iters)
+    if n_swaps[0] % 2:
+        swap()   # an even number of swaps: k and v end as they began
+    torch.cuda.synchronize()
     row = D * k.element_size()
     g_bytes = 4 * B * Hkv * S * row
     return {"ms_gather": round(t_g, 4), "ms_override": round(t_o, 4),
@@ -634,15 +645,16 @@ def kv_timing(api, torch, k, v, seeds, iters=20):
             "gbs_override": round(2 * g_bytes / (t_o * 1e-3) / 1e9, 1)}
 
 
-def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, pairs=200):
+def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, pairs=200, block_us=250.0):
     """Attention time with the configured seeds vs. the same tensors with no seeds.
 
-    `pairs` seeded / unseeded launches are interleaved (the order alternating from pair to pair),
-    each timed alone with CUDA events behind a device-side spin, so slow drifts of clock or
-    temperature hit both arms alike. The overhead is the median of the per-pair ratios, with
-    their 10th / 90th percentiles as its spread; the minimum and the median of each arm and the
-    ratio of the minima are reported beside it (on launches of ~15 us a single fast outlier
-    moves the minima by several percent, the pair median does not move).
+    `pairs` seeded / unseeded samples are interleaved (the order alternating from pair to pair),
+    each timed with CUDA events behind a device-side spin, so slow drifts of clock or
+    temperature hit both arms alike. A sample is a block of R back-to-back launches of one arm,
+    R chosen so that a block lasts about `block_us`: the event timestamps advance in steps of
+    ~1 us, which is 4-7 % of a single launch of the small shapes. The overhead is the median of
+    the per-pair ratios, with their 10th / 90th percentiles as its spread; the minimum and the
+    median of each arm and the ratio of the minima are reported beside it.
     """
     stream = torch.cuda.current_stream()
 
@@ -655,16 +667,27 @@ def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, pairs=2
     for _ in range(3):
         launch(True)
         launch(False)
+    one = []
+    for _ in range(5):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        busy_ahead(torch)
+        a.record(stream)
+        launch(True)
+        b.record(stream)
+        torch.cuda.synchronize()
+        one.append(a.elapsed_time(b))
+    R = max(1, min(16, round(block_us / (statistics.median(one) * 1e3))))
     ts = {True: [], False: []}
     for i in range(pairs):
         for with_seeds in ((True, False) if i % 2 == 0 else (False, True)):
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            busy_ahead(torch)
+            busy_ahead(torch, R)
             a.record(stream)
-            launch(with_seeds)
+            for _ in range(R):
+                launch(with_seeds)
             b.record(stream)
             torch.cuda.synchronize()
-            ts[with_seeds].append(a.elapsed_time(b))
+            ts[with_seeds].append(a.elapsed_time(b) / R)
     ratios = sorted(s / n - 1.0 for s, n in zip(ts[True], ts[False]))
     t_seed, t_none = min(ts[True]), min(ts[False])
     pct = lambda p: ratios[min(len(ratios) - 1, int(p * len(ratios)))]  # noqa: E731
@@ -676,7 +699,7 @@ def seed_overhead(api, torch, q, kc, vc, km, vm, seeds, out, lse, flops, pairs=2
             "overhead": round(statistics.median(ratios), 4),
             "overhead_p10_p90": [round(pct(0.1), 4), round(pct(0.9), 4)],
             "overhead_of_minima": round((t_seed - t_none) / t_none, 4),
-            "pairs": pairs}
+            "pairs": pairs, "launches_per_sample": R}
 
 
 # ----------------------------------------------------------------------------

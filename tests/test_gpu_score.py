@@ -61,10 +61,10 @@ def test_score_side_inputs_and_eligibility():
     check(inp, run_score(inp))
 
 
-@pytest.mark.parametrize("per,k", [(1000, 32), (300, 20)])
-def test_score_topk_fewer_eligible_than_k(per, k):
+@pytest.mark.parametrize("per,k,frac", [(1000, 32, 0.012), (300, 20, 0.012), (1000, 6, 0.003)])
+def test_score_topk_fewer_eligible_than_k(per, k, frac):
     """General path with fewer eligible rows than k: the list ends in -1 / -inf."""
-    inp = W.make_score_inputs(2 * per, 300, 2, k, seed=per, eligible_frac=0.012)
+    inp = W.make_score_inputs(2 * per, 300, 2, k, seed=per, eligible_frac=frac)
     r = run_score(inp)
     check(inp, r)
     n_elig = inp.eligible.reshape(2, per).sum(axis=1)
@@ -148,6 +148,8 @@ def test_score_named_workloads_full(name):
     (512, 1001, 33),    # the register-load kernel (512 threads): selection by rank
     (513, 1001, 32),    # and one row past it: warp sorts and merges
     (4096, 136, 32),    # the largest segment, k = 32
+    (600, 300, 9),      # the fewest keys taken by warp sorts
+    (600, 300, 8),      # the most taken by rounds of a CTA-wide maximum
     (777, 200, 1),      # k = 1
 ])
 def test_score_topk_on_both_sides_of_the_fast_path(per, V, k):
