@@ -349,19 +349,25 @@ def run_ours(args):
         stream.wait_stream(s_in)
         stream.wait_stream(s_out)
 
+    # three timed runs, the median reported: the host link is shared, and a run now and then
+    # takes ~20 % longer in every build, with or without any change on the device side
     e2e_steps = max(3, min(args.steps, 10))
     e2e_run(2)
     torch.cuda.synchronize()
-    barrier(ws)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    e2e_run(e2e_steps)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    barrier(ws)
-    e2e_ms = max_over_ranks(e0.elapsed_time(e1), ws) / e2e_steps
+    runs = []
+    for _ in range(3):
+        barrier(ws)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        e2e_run(e2e_steps)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier(ws)
+        runs.append(max_over_ranks(e0.elapsed_time(e1), ws) / e2e_steps)
+    e2e_ms = statistics.median(runs)
     e2e = {"value": round(ws * flops / (e2e_ms * 1e-3) / 1e12, 2), "unit": UNIT, "h2d_bytes_per_step": h2d,
            "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4),
+           "ms_per_step_runs": [round(r, 4) for r in runs], "steps_per_run": e2e_steps,
            "pipelined": "copy-in, compute and copy-out on three streams, double-buffered device tensors"}
     assert torch.equal(host_out["topk_idx"], sout["topk_idx"].cpu()), "e2e results differ from the device run"
     del dev_in, dev_out, host_in, host_out

@@ -18,6 +18,7 @@
 #include <stdint.h>
 
 #include "kernels.cuh"
+#include "ptx.cuh"
 
 namespace cover {
 namespace {
@@ -39,6 +40,10 @@ template <bool kOverride>
 __global__ void __launch_bounds__(kThreads) seed_kv_kernel(const KvParams p) {
   __shared__ int s_pos[kSlotsPerCta];
   __shared__ int s_dup[kSlotsPerCta];
+  // programmatic dependent launch: wait for the stream's previous kernel, let the next one be
+  // scheduled
+  griddep_wait();
+  griddep_launch_dependents();
   const int bh = blockIdx.x;               // b * Hkv + h
   const int b = bh / p.Hkv;
   const int slot0 = blockIdx.y * kSlotsPerCta;
@@ -111,11 +116,11 @@ int launch_seed_kv(bool override_swap, void* k, void* v, const int32_t* seed_idx
   KvParams p{static_cast<uint8_t*>(k), static_cast<uint8_t*>(v), seed_idx, n_seeds, L, Hkv, row_bytes / 16,
              static_cast<uint8_t*>(k_cache), static_cast<uint8_t*>(v_cache)};
   const dim3 grid(static_cast<unsigned>(bh), static_cast<unsigned>(chunks));
-  if (override_swap)
-    seed_kv_kernel<true><<<grid, kThreads, 0, stream>>>(p);
-  else
-    seed_kv_kernel<false><<<grid, kThreads, 0, stream>>>(p);
-  return cudaGetLastError() == cudaSuccess ? 0 : -3;
+  cudaLaunchAttribute attr[1];
+  const cudaLaunchConfig_t cfg = pdl_config(grid, dim3(kThreads), 0, stream, attr);
+  const cudaError_t e = override_swap ? cudaLaunchKernelEx(&cfg, seed_kv_kernel<true>, p)
+                                      : cudaLaunchKernelEx(&cfg, seed_kv_kernel<false>, p);
+  return e == cudaSuccess && cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
 
 }  // namespace cover

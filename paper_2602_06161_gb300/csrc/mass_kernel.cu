@@ -118,8 +118,10 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int hkv = hq / (Hq / Hkv);
   uint32_t* bits = col_bits(sm);
   float* colv = col_vals(sm, n_t);
-  // the reduction kernel behind this one may be scheduled now; it waits for this grid's results
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  // launched as a programmatic dependent of the stream's previous kernel: wait for its results;
+  // the reduction kernel behind this one may be scheduled now, it waits for this grid's results
+  griddep_wait();
+  griddep_launch_dependents();
 
   const CUtensorMap* tm_x = cols ? &tm_k : &tm_q;
   const CUtensorMap* tm_y = cols ? &tm_q : &tm_k;
@@ -339,7 +341,8 @@ __global__ void mass_reduce_kernel(const float* __restrict__ part_in, const floa
                                    int Hq, int per, float* __restrict__ d_in, float* __restrict__ d_out) {
   // launched as a programmatic dependent of mass_kernel: wait until its partial sums are complete
   // and visible
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  griddep_wait();
+  griddep_launch_dependents();
   const int n = blockIdx.x * blockDim.x + threadIdx.x;
   if (n >= B * per) return;
   const int b = n / per, i = n % per;
@@ -382,24 +385,22 @@ int launch_attn_mass(const MassArgs& a, int* status, cudaStream_t stream) {
   });
   if (rc != 0) return rc;
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
-  mass_kernel<<<dim3(static_cast<unsigned>(grid), 2), kThreads, smem, stream>>>(
-      tq, tk, static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.k_seedmask), a.seed_idx,
-      a.n_seeds, a.lse, a.Hq, a.Hkv, a.L, a.pos0, a.per, n_t, a.tok, a.flags, a.mask_id, scale_log2, part_in,
-      part_out, status);
+  {
+    cudaLaunchAttribute attr[1];
+    const cudaLaunchConfig_t cfg =
+        pdl_config(dim3(static_cast<unsigned>(grid), 2), dim3(kThreads), smem, stream, attr);
+    if (cudaLaunchKernelEx(&cfg, mass_kernel, tq, tk, static_cast<const __nv_bfloat16*>(a.q),
+                           static_cast<const __nv_bfloat16*>(a.k_seedmask), a.seed_idx, a.n_seeds, a.lse, a.Hq, a.Hkv,
+                           a.L, a.pos0, a.per, n_t, a.tok, a.flags, a.mask_id, scale_log2, part_in, part_out,
+                           status) != cudaSuccess)
+      return -3;
+  }
   if (cudaGetLastError() != cudaSuccess) return -3;
   // the reduction may launch while the partial sums are still being written (programmatic
   // dependent launch); it waits on the device for them, so its launch latency is hidden
   const int rows = a.B * a.per;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>((rows + 255) / 256));
-  cfg.blockDim = dim3(256);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = stream;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  const cudaLaunchConfig_t cfg = pdl_config(dim3(static_cast<unsigned>((rows + 255) / 256)), dim3(256), 0, stream, attr);
   return cudaLaunchKernelEx(&cfg, mass_reduce_kernel, static_cast<const float*>(part_in),
                             static_cast<const float*>(part_out), a.B, a.Hq, a.per, a.d_in, a.d_out) == cudaSuccess
              ? 0 : -3;

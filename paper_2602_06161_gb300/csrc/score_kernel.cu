@@ -1135,6 +1135,10 @@ __global__ void __launch_bounds__(kThreads, 2) score_kernel(const ScoreParams P)
   __shared__ int red_i[kWarps];
   __shared__ float2 red_z[kWarps], red_s[kWarps];
   __shared__ int s_last;
+  // programmatic dependent launch: wait for the stream's previous kernel, let the next one be
+  // scheduled
+  griddep_wait();
+  griddep_launch_dependents();
 
   const int n = blockIdx.x;
   const int tid = threadIdx.x;
@@ -1194,6 +1198,10 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
   __shared__ int red_i[kConsumerWarps + 1];
   __shared__ float2 red_z[kConsumerWarps + 1], red_s[kConsumerWarps + 1];
   __shared__ int s_last, s_abort;
+  // programmatic dependent launch: wait for the stream's previous kernel, let the next one be
+  // scheduled
+  griddep_wait();
+  griddep_launch_dependents();
 
   const int n = blockIdx.x;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -1297,6 +1305,10 @@ __global__ void __launch_bounds__(kSelectThreads) seed_select_kernel(const Decid
                                                                     const float* d_out, float* score, int per_seq,
                                                                     int sort_n) {
   extern __shared__ __align__(16) uint64_t sel_keys[];
+  // programmatic dependent launch: wait for the stream's previous kernel, let the next one be
+  // scheduled
+  griddep_wait();
+  griddep_launch_dependents();
   const int tid = threadIdx.x;
   if (per_seq <= static_cast<int>(blockDim.x)) {
     // one row per thread: the state in registers, selection by rank
@@ -1348,9 +1360,13 @@ int launch_score_impl(const ScoreArgs& a, const DecideArgs* d, int* status, cuda
                                   static_cast<int>(kRingStages * kChunkBytes)) == cudaSuccess ? 0 : -3;
     });
     if (rc != 0) return rc;
-    score_bulk_kernel<<<a.N, kBulkThreads, smem, stream>>>(P, status);
+    cudaLaunchAttribute attr[1];
+    const cudaLaunchConfig_t cfg = pdl_config(dim3(a.N), dim3(kBulkThreads), smem, stream, attr);
+    if (cudaLaunchKernelEx(&cfg, score_bulk_kernel, P, status) != cudaSuccess) return -3;
   } else {
-    score_kernel<<<a.N, kThreads, keys_bytes, stream>>>(P);
+    cudaLaunchAttribute attr[1];
+    const cudaLaunchConfig_t cfg = pdl_config(dim3(a.N), dim3(kThreads), keys_bytes, stream, attr);
+    if (cudaLaunchKernelEx(&cfg, score_kernel, P) != cudaSuccess) return -3;
   }
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
@@ -1372,7 +1388,9 @@ int launch_seed_select(int N, int n_seq, const DecideArgs& d, const float* d_in,
   while (sort_n < per) sort_n <<= 1;
   // at least one key per thread: the one-row-per-thread selection publishes up to 32 keys per warp
   const size_t smem = (sizeof(uint64_t) + sizeof(float)) * static_cast<size_t>(std::max(sort_n, kSelectThreads));
-  seed_select_kernel<<<n_seq, kSelectThreads, smem, stream>>>(d, d_in, d_out, score, per, sort_n);
+  cudaLaunchAttribute attr[1];
+  const cudaLaunchConfig_t cfg = pdl_config(dim3(n_seq), dim3(kSelectThreads), smem, stream, attr);
+  if (cudaLaunchKernelEx(&cfg, seed_select_kernel, d, d_in, d_out, score, per, sort_n) != cudaSuccess) return -3;
   return cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
 
