@@ -483,8 +483,10 @@ def decide_timing(api, torch, wl, iters=20):
     """Scoring fused with the decision step vs. scoring + top-k alone, on the same logits.
 
     Decision parameters follow the paper's setting (tau 0.9, budget B = 15,
-    ReMask budget 5); the decoding state is restored before every call, outside
-    the timed region. GB/s counts the logits read once plus the per-row state.
+    ReMask budget 5). Each sample times a block of R calls (R as in time_launches):
+    R consecutive decoding steps on the same logits, the state restored before the
+    block, outside the timed region. GB/s counts the logits read once plus the
+    per-row state.
     """
     di = wl.decide_inputs()
     per = di.N // di.n_seq
@@ -502,29 +504,38 @@ def decide_timing(api, torch, wl, iters=20):
     sout = api.cover_score_fwd(logits, di.n_seq, wl.score_topk, workspace=wsp)
     stream = torch.cuda.current_stream()
 
-    def timed(fused):
+    def timed(fused, R):
+        # a block of R calls: R consecutive decoding steps on the same logits for the fused call
+        # (the state, restored before each block, evolves from step to step as in decoding)
         ts = []
         for _ in range(iters):
             tok.copy_(tok0)
             flags.copy_(flags0)
             rc.copy_(rc0)
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            busy_ahead(torch)
+            busy_ahead(torch, R)
             a.record(stream)
-            if fused:
-                api.cover_score_decide_fwd(logits, di.n_seq, tok, flags, rc, workspace=ws, out=out, **kw)
-            else:
-                api.cover_score_fwd(logits, di.n_seq, wl.score_topk, workspace=wsp, out=sout)
+            for _ in range(R):
+                if fused:
+                    api.cover_score_decide_fwd(logits, di.n_seq, tok, flags, rc, workspace=ws, out=out, **kw)
+                else:
+                    api.cover_score_fwd(logits, di.n_seq, wl.score_topk, workspace=wsp, out=sout)
             b.record(stream)
             torch.cuda.synchronize()
-            ts.append(a.elapsed_time(b))
+            ts.append(a.elapsed_time(b) / R)
         return statistics.median(ts)
 
-    t_dec, t_score = timed(True), timed(False)
-    t_dec, t_score = min(t_dec, timed(True)), min(t_score, timed(False))
+    R = max(1, min(16, round(250.0 / (timed(False, 1) * 1e3))))
+    t_dec, t_score = timed(True, R), timed(False, R)
+    t_dec, t_score = min(t_dec, timed(True, R)), min(t_score, timed(False, R))
+    # the statistics below are those of the first step of a block
+    tok.copy_(tok0)
+    flags.copy_(flags0)
+    rc.copy_(rc0)
+    api.cover_score_decide_fwd(logits, di.n_seq, tok, flags, rc, workspace=ws, out=out, **kw)
     stats = out["stats"].cpu().numpy()
     nbytes = di.N * di.V * 2 + di.N * (20 + 12) + di.n_seq * wl.score_topk * 4
-    return {"ms_decide": round(t_dec, 4), "ms_score_topk": round(t_score, 4),
+    return {"ms_decide": round(t_dec, 4), "ms_score_topk": round(t_score, 4), "calls_per_sample": R,
             "overhead": round((t_dec - t_score) / t_score, 4),
             "gbs": round(nbytes / (t_dec * 1e-3) / 1e9, 1),
             "drafted_per_seq": round(float(stats[:, 0].mean()), 2),

@@ -55,7 +55,11 @@ constexpr int kChunkBytes = kChunkElems * 2;
 constexpr int kRingStages = 3;
 constexpr int kVecPerThread = kChunkElems / 8 / (kConsumerWarps * 32);   // 4
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr int kRoundsMax = 32;             // selections up to this size by rounds or warp sorts (top_select)
+constexpr int kMaxPerSeq = 4096;            // rows per segment (the entry points refuse more)
+constexpr int kRowLoads = 4;                // rows whose state a thread loads at once (general paths)
+constexpr int kRoundsMax = 32;
+constexpr int kRoundsFew = 8;               // selections up to this size by per-warp rounds (top_rounds)
+constexpr int kMaxWarps = 16;               // every kernel here runs at most 512 threads             // selections up to this size by rounds or warp sorts (top_select)
 
 struct RowAcc {
   float m;     // running maximum logit of this thread's elements
@@ -425,14 +429,24 @@ __device__ __forceinline__ int count_above(const uint64_t* l, uint64_t x) {
   return c;
 }
 
-// The k largest of the n keys in shared memory (keys are distinct, 0 = none), in descending
-// order, by k rounds of a CTA-wide maximum below the previous round's: one barrier per round,
-// the keys untouched. out[t] gets round t's key (0 once the nonzero keys run out). All threads
-// call it with the same k. Cheaper than top_warps for a few keys (about 0.65 us a round over
-// 1024 keys against about 5 us for the warp sorts).
+// Largest of the warp's 64-bit values (two 32-bit reductions: the high words, then the low
+// words of the lanes that hold the largest high word).
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t x) {
+  const uint32_t hi = __reduce_max_sync(0xffffffffu, static_cast<uint32_t>(x >> 32));
+  const uint32_t lo = __reduce_max_sync(0xffffffffu, static_cast<uint32_t>(x >> 32) == hi ? static_cast<uint32_t>(x) : 0u);
+  return (static_cast<uint64_t>(hi) << 32) | lo;
+}
+
+// The k largest (k <= kRoundsFew) of the n keys in shared memory (keys are distinct, 0 = none),
+// in descending order: out[t] gets the t-th (0 once the nonzero keys run out). Each warp takes
+// its own k largest by k rounds of a warp-wide maximum below the previous round's (no block
+// barrier per round), over the keys its lanes read (i = tid, tid + blockDim, ...); a key can be
+// among the k largest only if it is among its warp's, so ranking the warps' lists against each
+// other is exact below k. All threads call it with the same k.
 __device__ __forceinline__ void top_rounds(const uint64_t* keys, int n, int k, uint64_t* out) {
-  __shared__ unsigned long long s_max[2][32];
+  __shared__ uint64_t s_list[kMaxWarps * kRoundsFew];
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31, warp = tid >> 5, nw = nt >> 5;
+  if (k <= 0) return;
   uint64_t prev = ~0ull;
   for (int t = 0; t < k; ++t) {
     uint64_t m = 0;
@@ -440,22 +454,19 @@ __device__ __forceinline__ void top_rounds(const uint64_t* keys, int n, int k, u
       const uint64_t x = keys[i];
       if (x < prev && x > m) m = x;
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const uint64_t y = __shfl_xor_sync(0xffffffffu, m, o);
-      m = y > m ? y : m;
-    }
-    if (lane == 0) s_max[t & 1][warp] = m;
-    __syncthreads();
-    m = 0;
-    for (int w = 0; w < nw; ++w) m = s_max[t & 1][w] > m ? s_max[t & 1][w] : m;
-    if (tid == 0) out[t] = m;
-    prev = m;
-    if (m == 0) {
-      for (int r = t + 1 + tid; r < k; r += nt) out[r] = 0;
-      break;
-    }
+    prev = warp_max_u64(m);
+    if (lane == 0) s_list[warp * k + t] = prev;   // 0 once the warp's keys run out
   }
+  const int nl = nw * k;
+  __syncthreads();
+  const uint64_t key = tid < nl ? s_list[tid] : 0;
+  const int listed = __syncthreads_count(key != 0);
+  if (key != 0) {
+    int r = 0;
+    for (int j = 0; j < nl; ++j) r += s_list[j] > key ? 1 : 0;
+    if (r < k) out[r] = key;
+  }
+  for (int t = min(listed, k) + tid; t < k; t += nt) out[t] = 0;
   __syncthreads();
 }
 
@@ -508,7 +519,6 @@ __device__ __forceinline__ void top_warps(uint64_t* keys, int n, int k, uint64_t
 
 // The k largest (k <= kRoundsMax) of n keys in shared memory into out, by rounds for a few keys
 // and by warp sorts otherwise; the first 32 * warps keys may be overwritten.
-constexpr int kRoundsFew = 8;
 __device__ __forceinline__ void top_select(uint64_t* keys, int n, int k, uint64_t* out) {
   if (k <= kRoundsFew)
     top_rounds(keys, n, k, out);
@@ -524,6 +534,7 @@ __device__ __forceinline__ void top_select(uint64_t* keys, int n, int k, uint64_
 // runs only when more rows pass the threshold than the budget allows.
 __device__ void segment_update(uint64_t* keys, int seg, int per_seq, int sort_n, const ScoreParams& P) {
   __shared__ unsigned long long s_fallback;
+  __shared__ uint32_t s_draft_bits[kMaxPerSeq / 32];
   __shared__ int s_ri[32];
   __shared__ int s_cnt[3][32];
   __shared__ uint64_t s_sel[kRoundsMax];
@@ -533,18 +544,39 @@ __device__ void segment_update(uint64_t* keys, int seg, int per_seq, int sort_n,
   if (tid == 0) s_fallback = ~0ull;
   __syncthreads();
 
-  // Section 5.2 drafting: masked rows in the allowed set whose confidence exceeds tau
+  // Section 5.2 drafting: masked rows in the allowed set whose confidence exceeds tau. Each
+  // thread loads the state of kRowLoads rows before it uses any of it (the loads of a batch
+  // overlap instead of waiting on one another's results).
   int ncand = 0;
-  for (int i = tid; i < per_seq; i += nt) {
-    const int n = base + i;
-    if (d.tok[n] == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0)) {
-      if (__ldcg(P.maxprob + n) > d.tau) ++ncand;
-      if (d.min_one) {
-        // lowest entropy, then lowest index
-        const uint64_t fb = (static_cast<uint64_t>(order_key(__ldcg(P.entropy + n))) << 32) | static_cast<uint32_t>(i);
-        atomicMin(&s_fallback, static_cast<unsigned long long>(fb));
-      }
+  uint64_t fb_min = ~0ull;   // the thread's lowest (entropy, index) key among allowed rows
+  for (int i0 = tid; i0 < per_seq; i0 += kRowLoads * nt) {
+    bool allowed[kRowLoads];
+    float c[kRowLoads], h[kRowLoads];
+#pragma unroll
+    for (int u = 0; u < kRowLoads; ++u) {
+      const int i = i0 + u * nt;
+      const bool in = i < per_seq;
+      const int n = base + (in ? i : 0);
+      allowed[u] = in && d.tok[n] == d.mask_id & (d.draft_ok == nullptr || d.draft_ok[n] != 0);
+      c[u] = __ldcg(P.maxprob + n);
+      h[u] = __ldcg(P.entropy + n);
     }
+#pragma unroll
+    for (int u = 0; u < kRowLoads; ++u) {
+      if (!allowed[u]) continue;
+      if (c[u] > d.tau) ++ncand;
+      // lowest entropy, then lowest index
+      const uint64_t fb = (static_cast<uint64_t>(order_key(h[u])) << 32) | static_cast<uint32_t>(i0 + u * nt);
+      fb_min = fb < fb_min ? fb : fb_min;
+    }
+  }
+  if (d.min_one) {
+    // one shared-memory atomic per warp (a 64-bit minimum by two 32-bit reductions)
+    const uint32_t hi = __reduce_min_sync(0xffffffffu, static_cast<uint32_t>(fb_min >> 32));
+    const uint32_t lo =
+        __reduce_min_sync(0xffffffffu, static_cast<uint32_t>(fb_min >> 32) == hi ? static_cast<uint32_t>(fb_min) : ~0u);
+    const uint64_t wmin = (static_cast<uint64_t>(hi) << 32) | lo;   // ~0 only when no lane has a row
+    if (lane == 0 && wmin != ~0ull) atomicMin(&s_fallback, static_cast<unsigned long long>(wmin));
   }
   ncand = block_sum(ncand, s_ri);
   const bool all_cand = ncand <= d.budget;   // every row above tau is drafted
@@ -552,14 +584,22 @@ __device__ void segment_update(uint64_t* keys, int seg, int per_seq, int sort_n,
   const bool fallback = n_drafted == 0 && d.min_one && s_fallback != ~0ull;
   if (!all_cand) {
     // more candidates than the budget: the `budget` most confident (ties to the lower index)
-    for (int i = tid; i < sort_n; i += nt) {
-      uint64_t key = 0;
-      if (i < per_seq) {
-        const int n = base + i;
-        const float c = __ldcg(P.maxprob + n);
-        if (d.tok[n] == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0) && c > d.tau) key = rank_key(c, i);
+    for (int i0 = tid; i0 < sort_n; i0 += kRowLoads * nt) {
+      bool allowed[kRowLoads];
+      float c[kRowLoads];
+#pragma unroll
+      for (int u = 0; u < kRowLoads; ++u) {
+        const int i = i0 + u * nt;
+        const bool in = i < per_seq;
+        const int n = base + (in ? i : 0);
+        allowed[u] = in && d.tok[n] == d.mask_id & (d.draft_ok == nullptr || d.draft_ok[n] != 0);
+        c[u] = __ldcg(P.maxprob + n);
       }
-      keys[i] = key;
+#pragma unroll
+      for (int u = 0; u < kRowLoads; ++u) {
+        const int i = i0 + u * nt;
+        if (i < sort_n) keys[i] = allowed[u] && c[u] > d.tau ? rank_key(c[u], i) : 0;
+      }
     }
     __syncthreads();
     if (n_drafted <= kRoundsMax)
@@ -567,43 +607,64 @@ __device__ void segment_update(uint64_t* keys, int seg, int per_seq, int sort_n,
     else
       bitonic_sort_desc(keys, sort_n);
   }
+  // the drafted rows, marked for the pass below when they were selected (more candidates than
+  // the budget) or are the fallback row; with every candidate drafted the pass decides itself
   if (!all_cand || fallback) {
+    for (int w = tid; w < kMaxPerSeq / 32; w += nt) s_draft_bits[w] = 0u;
+    __syncthreads();
     const uint64_t* picked = n_drafted <= kRoundsMax ? s_sel : keys;
     for (int t = tid; t < (fallback ? 1 : n_drafted); t += nt) {
-      const int n = base + (fallback ? static_cast<int>(static_cast<uint32_t>(s_fallback)) : rank_key_row(picked[t]));
-      // a drafted row takes its greedy token, whose uncertainty is ln Z
-      d.tok[n] = __ldcg(P.argmax + n);
-      d.ws_u[n] = __ldcg(d.ws_lnz + n);
-      d.flags[n] = static_cast<uint8_t>((d.flags[n] & ~1u) | 2u);
+      const int i = fallback ? static_cast<int>(static_cast<uint32_t>(s_fallback)) : rank_key_row(picked[t]);
+      atomicOr(&s_draft_bits[i >> 5], 1u << (i & 31));
     }
     __syncthreads();
   }
+  const bool marked = !all_cand || fallback;
   if (fallback) n_drafted = 1;
 
   // Section 5.2 revision of the previous seeds, Section 3 state update
   int kept = 0, replaced = 0, remasked = 0;
-  for (int i = tid; i < per_seq; i += nt) {
-    const int n = base + i;
-    const int y = d.tok[n];
-    const uint8_t fl = d.flags[n];
-    if (all_cand && y == d.mask_id && (d.draft_ok == nullptr || d.draft_ok[n] != 0) &&
-        __ldcg(P.maxprob + n) > d.tau) {
-      // drafted (every candidate fits the budget)
-      d.tok[n] = __ldcg(P.argmax + n);
-      d.ws_u[n] = __ldcg(d.ws_lnz + n);
-      d.flags[n] = static_cast<uint8_t>((fl & ~1u) | 2u);
-    } else if ((fl & 1u) != 0 && y != d.mask_id) {
-      const int yh = __ldcg(P.argmax + n);
-      if (yh == y) {
-        ++kept;
-      } else if (__ldcg(P.maxprob + n) > d.tau) {
-        ++replaced;
-        d.tok[n] = yh;
-        d.ws_u[n] = __ldcg(d.ws_lnz + n);
-      } else {
-        ++remasked;
-        d.tok[n] = d.mask_id;
-        d.remask_cnt[n] = static_cast<uint8_t>(min(d.remask_cnt[n] + 1, 255));
+  for (int i0 = tid; i0 < per_seq; i0 += kRowLoads * nt) {
+    int y[kRowLoads], yh[kRowLoads];
+    uint32_t fl[kRowLoads], rc[kRowLoads];
+    bool ok[kRowLoads];
+    float c[kRowLoads], lz[kRowLoads];
+#pragma unroll
+    for (int u = 0; u < kRowLoads; ++u) {
+      const int i = i0 + u * nt;
+      const int n = base + (i < per_seq ? i : 0);
+      y[u] = d.tok[n];
+      fl[u] = d.flags[n];
+      rc[u] = d.remask_cnt[n];
+      ok[u] = d.draft_ok == nullptr || d.draft_ok[n] != 0;
+      c[u] = __ldcg(P.maxprob + n);
+      yh[u] = __ldcg(P.argmax + n);
+      lz[u] = __ldcg(d.ws_lnz + n);
+    }
+#pragma unroll
+    for (int u = 0; u < kRowLoads; ++u) {
+      const int i = i0 + u * nt;
+      if (i >= per_seq) continue;
+      const int n = base + i;
+      const bool drafted = marked ? (s_draft_bits[i >> 5] >> (i & 31)) & 1u
+                                  : y[u] == d.mask_id && ok[u] && c[u] > d.tau;
+      if (drafted) {
+        // a drafted row takes its greedy token, whose uncertainty is ln Z
+        d.tok[n] = yh[u];
+        d.ws_u[n] = lz[u];
+        d.flags[n] = static_cast<uint8_t>((fl[u] & ~1u) | 2u);
+      } else if ((fl[u] & 1u) != 0 && y[u] != d.mask_id) {
+        if (yh[u] == y[u]) {
+          ++kept;
+        } else if (c[u] > d.tau) {
+          ++replaced;
+          d.tok[n] = yh[u];
+          d.ws_u[n] = lz[u];
+        } else {
+          ++remasked;
+          d.tok[n] = d.mask_id;
+          d.remask_cnt[n] = static_cast<uint8_t>(min(rc[u] + 1u, 255u));
+        }
       }
     }
   }
@@ -652,28 +713,45 @@ __device__ void segment_select(uint64_t* keys, int seg, int per_seq, int sort_n,
 
   int n_t = 0;
   uint32_t emax = 0;   // largest biased exponent of the finite scores
-  for (int i = tid; i < sort_n; i += nt) {
-    uint64_t key = 0;
-    if (i < per_seq) {
-      const int n = base + i;
-      const uint8_t fl = d.flags[n];
-      float s = -INFINITY;
-      if (d.tok[n] != d.mask_id) {
-        const float din = d_in != nullptr ? d_in[n] : 0.0f;
-        const float dout = d_out != nullptr ? d_out[n] : 0.0f;
-        const float sc = __ldcg(d.ws_u + n) * (1.0f + din) / (1.0f + dout);
-        if (isfinite(sc)) {
-          s = sc;
-          ++n_t;
-          emax = max(emax, (__float_as_uint(sc) >> 23) & 0xffu);
-          if ((fl & 1u) == 0 && d.remask_cnt[n] < d.remask_budget) key = rank_key(sc, i);
-        }
-      }
-      score[n] = s;
-      sscore[i] = s;
-      d.flags[n] = static_cast<uint8_t>(fl & ~3u);
+  for (int i0 = tid; i0 < sort_n; i0 += kRowLoads * nt) {
+    // the state of kRowLoads rows, loaded before any of it is used
+    uint32_t fl[kRowLoads], rc[kRowLoads];
+    int tk[kRowLoads];
+    float din[kRowLoads], dout[kRowLoads], uu[kRowLoads];
+#pragma unroll
+    for (int u = 0; u < kRowLoads; ++u) {
+      const int i = i0 + u * nt;
+      const int n = base + (i < per_seq ? i : 0);
+      fl[u] = d.flags[n];
+      rc[u] = d.remask_cnt[n];
+      tk[u] = d.tok[n];
+      din[u] = d_in != nullptr ? d_in[n] : 0.0f;
+      dout[u] = d_out != nullptr ? d_out[n] : 0.0f;
+      uu[u] = __ldcg(d.ws_u + n);
     }
-    keys[i] = key;
+#pragma unroll
+    for (int u = 0; u < kRowLoads; ++u) {
+      const int i = i0 + u * nt;
+      if (i >= sort_n) continue;
+      uint64_t key = 0;
+      if (i < per_seq) {
+        const int n = base + i;
+        float s = -INFINITY;
+        if (tk[u] != d.mask_id) {
+          const float sc = uu[u] * (1.0f + din[u]) / (1.0f + dout[u]);
+          if (isfinite(sc)) {
+            s = sc;
+            ++n_t;
+            emax = max(emax, (__float_as_uint(sc) >> 23) & 0xffu);
+            if ((fl[u] & 1u) == 0 && static_cast<int>(rc[u]) < d.remask_budget) key = rank_key(sc, i);
+          }
+        }
+        score[n] = s;
+        sscore[i] = s;
+        d.flags[n] = static_cast<uint8_t>(fl[u] & ~3u);
+      }
+      keys[i] = key;
+    }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) n_t += __shfl_xor_sync(0xffffffffu, n_t, o);
@@ -1301,6 +1379,8 @@ __global__ void __launch_bounds__(kBulkThreads, 4) score_bulk_kernel(const Score
 // Section 5.3 selection as its own launch (one CTA per segment), after the
 // update phase and the d_in / d_out pass.
 constexpr int kSelectThreads = 512;
+static_assert(kThreads <= 32 * kMaxWarps && kBulkThreads <= 32 * kMaxWarps && kSelectThreads <= 32 * kMaxWarps,
+              "top_rounds keeps a list per warp for at most kMaxWarps warps");
 __global__ void __launch_bounds__(kSelectThreads) seed_select_kernel(const DecideArgs d, const float* d_in,
                                                                     const float* d_out, float* score, int per_seq,
                                                                     int sort_n) {
