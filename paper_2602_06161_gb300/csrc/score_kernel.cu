@@ -1007,9 +1007,16 @@ __device__ void decide_fast(uint64_t* keys, int seg, int per_seq, const ScorePar
   // Section 5.2 drafting: masked rows in the allowed set whose confidence exceeds tau
   const bool allowed = in && tok == d.mask_id && ok_draft;
   const bool cand = allowed && c > d.tau;
-  if (d.min_one && allowed)   // lowest entropy, then lowest index
-    atomicMin(&s_fallback, static_cast<unsigned long long>((static_cast<uint64_t>(order_key(H)) << 32) |
-                                                            static_cast<uint32_t>(tid)));
+  if (d.min_one) {
+    // lowest entropy, then lowest index: a warp minimum (two 32-bit reductions), then one
+    // shared-memory atomic per warp
+    const uint64_t fb = allowed ? (static_cast<uint64_t>(order_key(H)) << 32) | static_cast<uint32_t>(tid) : ~0ull;
+    const uint32_t hi = __reduce_min_sync(0xffffffffu, static_cast<uint32_t>(fb >> 32));
+    const uint32_t lo =
+        __reduce_min_sync(0xffffffffu, static_cast<uint32_t>(fb >> 32) == hi ? static_cast<uint32_t>(fb) : ~0u);
+    const uint64_t wmin = (static_cast<uint64_t>(hi) << 32) | lo;   // ~0 only when no lane has a row
+    if (lane == 0 && wmin != ~0ull) atomicMin(&s_fallback, static_cast<unsigned long long>(wmin));
+  }
   const int ncand = __syncthreads_count(cand);
   const bool all_cand = ncand <= d.budget;   // every row above tau is drafted
   int n_drafted = min(ncand, d.budget);
