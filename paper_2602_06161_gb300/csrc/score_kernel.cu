@@ -1451,6 +1451,16 @@ int launch_score_impl(const ScoreArgs& a, const DecideArgs* d, int* status, cuda
     const cudaLaunchConfig_t cfg = pdl_config(dim3(a.N), dim3(kBulkThreads), smem, stream, attr);
     if (cudaLaunchKernelEx(&cfg, score_bulk_kernel, P, status) != cudaSuccess) return -3;
   } else {
+    // decision keys of the longest segment: 4096 x 12 bytes, above the 48 KB a launch gets
+    // without opting in (with the static shared memory)
+    static ContextCache<int> setup_reg;
+    int unused = 0;
+    const int rc = setup_reg.get(&unused, [](int&) {
+      return cudaFuncSetAttribute(score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>((sizeof(uint64_t) + sizeof(float)) * kMaxPerSeq)) == cudaSuccess
+                 ? 0 : -3;
+    });
+    if (rc != 0) return rc;
     cudaLaunchAttribute attr[1];
     const cudaLaunchConfig_t cfg = pdl_config(dim3(a.N), dim3(kThreads), keys_bytes, stream, attr);
     if (cudaLaunchKernelEx(&cfg, score_kernel, P) != cudaSuccess) return -3;
@@ -1475,6 +1485,15 @@ int launch_seed_select(int N, int n_seq, const DecideArgs& d, const float* d_in,
   while (sort_n < per) sort_n <<= 1;
   // at least one key per thread: the one-row-per-thread selection publishes up to 32 keys per warp
   const size_t smem = (sizeof(uint64_t) + sizeof(float)) * static_cast<size_t>(std::max(sort_n, kSelectThreads));
+  // the longest segment's keys and scores (48 KB) need the opt-in above the default limit
+  static ContextCache<int> setup;
+  int unused = 0;
+  const int rc = setup.get(&unused, [](int&) {
+    return cudaFuncSetAttribute(seed_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>((sizeof(uint64_t) + sizeof(float)) * kMaxPerSeq)) == cudaSuccess
+               ? 0 : -3;
+  });
+  if (rc != 0) return rc;
   cudaLaunchAttribute attr[1];
   const cudaLaunchConfig_t cfg = pdl_config(dim3(n_seq), dim3(kSelectThreads), smem, stream, attr);
   if (cudaLaunchKernelEx(&cfg, seed_select_kernel, d, d_in, d_out, score, per, sort_n) != cudaSuccess) return -3;

@@ -184,24 +184,28 @@ def test_decide_named_workload_full():
 
 
 @pytest.mark.parametrize("per,V", [
-    (288, 1000),   # one row per thread of the bulk-copy kernel (288 threads): the fast path
-    (289, 1000),   # one row more than its threads: the general path
-    (512, 1001),   # the register-load kernel (odd vocabulary, 512 threads): its fast-path limit
-    (513, 1001),   # and one row past it
+    (288, 1000),    # one row per thread of the bulk-copy kernel (288 threads): the fast path
+    (289, 1000),    # one row more than its threads: the general path
+    (1153, 1000),   # the general path, four rows per thread and one more
+    (512, 1001),    # the register-load kernel (odd vocabulary, 512 threads): its fast-path limit
+    (513, 1001),    # and one row past it
+    (2049, 1001),   # a segment of 2049 rows: 48 KB of keys and scores in shared memory
 ])
 def test_decide_both_sides_of_the_fast_path(per, V):
     # the per-sequence decision has a one-row-per-thread path and a general one; on both sides
     # of the switch the decisions equal the oracle's, with a drafting budget that forces the
-    # ranking (more candidates than the budget) and a seed cap above 32 (sort instead of rounds)
+    # ranking (more candidates than the budget) and a seed cap above 32 (rank or sort instead of
+    # the short selections)
     di = W.make_decide_inputs(2 * per, V, 2, seed=per, block_len=64)
     for p in (_params(draft_budget=15, max_seeds=8), _params(draft_budget=2, tau_draft=0.05, max_seeds=40)):
         check(di, p, run_decide(di, p), what=f"per {per} V {V} B {p['draft_budget']}")
 
 
-@pytest.mark.parametrize("per", [256, 512, 513, 1024])
+@pytest.mark.parametrize("per", [256, 512, 513, 1024, 2049])
 def test_update_then_select_both_paths(per):
     # the split order (update phase, then the selection launch with the caller's d_in / d_out):
-    # the selection launch has 512 threads, so 512 rows take its fast path and 513 the general one
+    # the selection launch has 512 threads, so 512 rows take its fast path and 513 the general
+    # one; 2049 rows need 48 KB of shared memory for the keys and scores
     di = W.make_decide_inputs(2 * per, 1000, 2, seed=per + 1, block_len=32)
     p = _params(max_seeds=12)
     logits = H.to_dev(di.logits, "bf16")
