@@ -235,6 +235,23 @@ def _dev_inputs(inp):
             H.to_dev(inp.k_seedmask, "bf16"), H.to_dev(inp.v_seedmask, "bf16"), H.to_dev(inp.seed_idx, "i32")]
 
 
+def test_bf16_dominant_self_term():
+    """Seed rows whose masked self score lies far above the row's other scores: the self term's
+    weight relative to the running maximum is ~2^45 for some rows and 2^140 to 2^175 for others
+    (beyond the bf16 range of the probabilities P; the merge rescales O instead)."""
+    inp = W.make_attn_inputs(1, 2, 1, 384, 128, 12, dtype="bf16", seed=5)
+    q = W.bf16_bits_to_f32(inp.q)
+    km = W.bf16_bits_to_f32(inp.k_seedmask)
+    for s, i in enumerate(inp.seed_idx[0]):
+        lam = 35.0 if s % 2 == 0 else 115.0
+        # head 0's query of row i sets the direction; the masked key is shared by both query heads
+        km[0, 0, s] = q[0, 0, i] / np.linalg.norm(q[0, 0, i]) * lam
+    inp.k_seedmask = W.f32_to_bf16_bits(km)
+    out, lse = H.run_attn(inp)
+    ref, ref_lse = H.oracle_full(inp)
+    H.assert_bf16_close(out, ref, lse, ref_lse)
+
+
 def test_bf16_invariances_bit_exact():
     inp = W.make_attn_inputs(2, 4, 2, 640, 128, 24, dtype="bf16", seed=21)
     args = _dev_inputs(inp)
