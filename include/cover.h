@@ -16,6 +16,11 @@
  *    The library allocates no device memory and keeps no per-call state.
  *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
  *    stream). Argument errors are returned synchronously, before any launch.
+ *  - Every kernel is launched as a programmatic dependent of the stream's
+ *    previous kernel: its CTAs may start while that kernel finishes, but they
+ *    read and write no global memory before it has completed and its writes
+ *    are visible, so stream order holds as for plain launches. Work after an
+ *    event wait or a copy on the stream is ordered as usual.
  *  - Kernels never trap. A kernel that gives up on an internal wait (bounded at
  *    about one second) records COVER_ERR_DEVICE_TIMEOUT in a per-device status
  *    word; read and clear it with cover_device_status().
