@@ -151,6 +151,7 @@ def test_score_named_workloads_full(name):
     (600, 300, 9),      # the fewest keys taken by warp sorts
     (600, 300, 8),      # the most taken by rounds of a CTA-wide maximum
     (777, 200, 1),      # k = 1
+    (600, 1001, 5),     # the register-load kernel's general path (16 warps), rounds
 ])
 def test_score_topk_on_both_sides_of_the_fast_path(per, V, k):
     inp = W.make_score_inputs(2 * per, V, 2, k, seed=per + k, spike_frac=0.1, eligible_frac=0.8)
