@@ -59,7 +59,7 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-secondary", action="store_true")
-    ap.add_argument("--only", choices=["attn", "prefix", "score", "decide", "mass"], default=None,
+    ap.add_argument("--only", choices=["attn", "prefix", "score", "decide", "mass", "kv"], default=None,
                     help="time one kernel alone on the workload (for profiler captures)")
     return ap.parse_args()
 
@@ -864,6 +864,13 @@ def run_only(args):
         tok, flags = torch.from_numpy(di.tok).cuda(), torch.from_numpy(di.flags | 2 * di.draft_ok).cuda()
         fn = lambda: api.cover_attn_mass_fwd(  # noqa: E731
             q, kc, lse, tok, flags, mask_id=di.mask_id, pos0=wl.L - per, per=per, k_seedmask=km, seed_idx=seeds)
+    elif args.only == "kv":
+        # the per-layer override swap of the seed K/V cache (after one gather that fills the cache)
+        ai = wl.attn_inputs()
+        kc, vc = bf16_dev(ai.k_cached, torch), bf16_dev(ai.v_cached, torch)
+        seeds = torch.from_numpy(ai.seed_idx).cuda()
+        kcache, vcache = api.cover_seed_kv_gather(kc, vc, seeds)
+        fn = lambda: api.cover_seed_kv_override(kc, vc, seeds, kcache, vcache)  # noqa: E731
     else:
         di = wl.decide_inputs()
         logits = bf16_dev(di.logits, torch)
