@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libcover.so")
 
-SOURCES = ["cover_api.cu", "context.cu", "tmap.cu", "route_kernel.cu", "attn_f32.cu", "attn_bf16_sm103.cu",
+SOURCES = ["cover_api.cu", "context.cu", "tmap.cu", "route_kernel.cu", "attn_f32.cu", "attn_bf16_sm103.cu", "attn_window_gqa.cu",
            "score_kernel.cu", "kv_kernel.cu", "mass_kernel.cu", "debug_kernels.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]

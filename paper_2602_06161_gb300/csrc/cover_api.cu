@@ -96,6 +96,7 @@ int cover_attn_fwd_prefix(const void* q, const void* k_cached, const void* v_cac
   if (st == nullptr) return COVER_ERR_CUDA;
   cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
                     Lq, q0};
+  if (cover::window_gqa_applies(a)) return cover::launch_attn_window_gqa(a, st, static_cast<cudaStream_t>(stream));
   return cover::launch_attn_bf16_sm103(a, st, static_cast<cudaStream_t>(stream));
 }
 

@@ -29,6 +29,16 @@ struct AttnArgs {
 };
 
 int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream);
+
+// Prefix-cache windows of grouped-query heads (attn_window_gqa.cu): the G = Hq / Hkv query heads
+// of a KV head packed into common Q tiles, the keys split over a cluster of up to 8 CTAs. Taken
+// for a window (Lq != L or q0 != 0) with G >= 2, Lq <= kMaxWindowGqaRows,
+// G * Lq <= kMaxWindowGqaPacked and at most 8 * kMaxWindowGqaSteps KV tiles of 128 keys.
+constexpr int kMaxWindowGqaRows = 256;
+constexpr int kMaxWindowGqaPacked = 256;
+constexpr int kMaxWindowGqaSteps = 8;
+bool window_gqa_applies(const AttnArgs& a);
+int launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream);
 int launch_attn_f32(const AttnArgs& a, int* status, cudaStream_t stream);
 
 int launch_seed_route(const int32_t* seed_idx, int n_seeds, int B, int L, int32_t* slot_out, uint32_t* bitmap_out,

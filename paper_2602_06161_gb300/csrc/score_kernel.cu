@@ -57,9 +57,9 @@ constexpr int kVecPerThread = kChunkElems / 8 / (kConsumerWarps * 32);   // 4
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kMaxPerSeq = 4096;            // rows per segment (the entry points refuse more)
 constexpr int kRowLoads = 4;                // rows whose state a thread loads at once (general paths)
-constexpr int kRoundsMax = 32;
+constexpr int kRoundsMax = 32;              // selections up to this size by rounds or warp sorts (top_select)
 constexpr int kRoundsFew = 8;               // selections up to this size by per-warp rounds (top_rounds)
-constexpr int kMaxWarps = 16;               // every kernel here runs at most 512 threads             // selections up to this size by rounds or warp sorts (top_select)
+constexpr int kMaxWarps = 16;               // every kernel here runs at most 512 threads
 
 struct RowAcc {
   float m;     // running maximum logit of this thread's elements

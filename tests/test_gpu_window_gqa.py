@@ -1,0 +1,90 @@
+"""GPU parity of the packed grouped-query window kernel (the prefix-cache window of Section 6.6
+for G = Hq / Hkv >= 2 and G * Lq <= 256 packed rows) against the fp64 oracle.
+
+The kernel packs a KV head's G query heads into common 128-row Q tiles and splits the keys over
+the CTAs of a cluster (T = ceil(nkv / 8) KV tiles per CTA, nsplit = ceil(nkv / T) CTAs), which
+combine their partial (m, l, O) through distributed shared memory and merge a seed row's masked
+self term there. The cases below reach one and several KV steps per CTA, clusters of 1 to 8
+CTAs, one and two Q tiles, packed-row counts that end inside a 32-row warp, a ragged last KV
+tile, a seed whose diagonal is the only key of its split, and routing of repeated and
+out-of-range seed entries."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2602_06161_gb300 import api
+from paper_2602_06161_gb300 import workloads as W
+from tests import _gpu as H
+from tests.test_gpu_prefix import _case, run_window
+
+pytestmark = pytest.mark.gpu
+
+
+def _check(q, kc, vc, km, vm, seeds, q0, Lq):
+    out, lse = run_window(q, kc, vc, km, vm, seeds, q0, Lq, "bf16")
+    f = W.bf16_bits_to_f64
+    ref, ref_lse = oracle.override_attention_window(f(q[:, :, q0:q0 + Lq]), f(kc), f(vc), f(km), f(vm),
+                                                    seeds if seeds.shape[1] else None, q0)
+    d = np.abs(out - ref)
+    assert np.isfinite(out).all() and np.isfinite(lse).all()
+    assert d.max() <= H.TOL_BF16_MAX and d.mean() <= H.TOL_BF16_MEAN, (d.max(), d.mean())
+    assert np.abs(lse - ref_lse).max() <= H.TOL_LSE
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,Lk,Lq,q0,S,inside", [
+    (1, 28, 4, 1024, 32, 992, 32, 6),      # Dream active block at the end: 8 one-step CTAs, 2 Q tiles
+    (1, 28, 4, 1024, 32, 992, 0, 0),       # the same without seeds
+    (1, 8, 2, 1100, 20, 1080, 12, 5),      # 9 KV tiles: 5 CTAs of 2, 1 steps; ragged tail holds diagonals
+    (1, 8, 2, 8192, 32, 8160, 16, 8),      # 64 KV tiles: 8 CTAs of 8 steps each
+    (1, 4, 2, 700, 128, 300, 10, 6),       # 256 packed rows (the limit), window in the middle
+    (2, 9, 3, 333, 37, 100, 7, 3),         # 111 packed rows: the last warp's rows end mid-warp
+    (1, 16, 2, 640, 16, 624, 5, 2),        # G = 8: one full Q tile
+    (3, 10, 5, 90, 3, 40, 4, 2),           # one ragged KV tile: a cluster of one CTA
+])
+def test_packed_window_matches_oracle(B, Hq, Hkv, Lk, Lq, q0, S, inside):
+    q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, S, q0, Lq, "bf16", 3 * Lk + Lq, inside)
+    _check(q, kc, vc, km, vm, seeds, q0, Lq)
+
+
+def test_packed_window_seed_alone_in_its_split():
+    # Lk = 129: the second KV tile holds one key, position 128, which is the window's row and a
+    # seed; its cached diagonal is excluded, so that split has no key left for the row and the
+    # combine must take the row from the other split and the masked self term alone
+    B, Hq, Hkv, Lk, Lq, q0 = 2, 6, 2, 129, 1, 128
+    q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, 3, q0, Lq, "bf16", 41, 1)
+    assert all(128 in seeds[b] for b in range(B))
+    _check(q, kc, vc, km, vm, seeds, q0, Lq)
+
+
+def test_packed_window_repeated_and_out_of_range_seeds():
+    # a position named by two slots takes the lower slot's masked row; entries outside [0, Lk)
+    # are ignored
+    B, Hq, Hkv, Lk, Lq, q0, S = 2, 12, 4, 520, 40, 480, 10
+    q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, S, q0, Lq, "bf16", 57, 5)
+    for b in range(B):
+        inside = [s for s in seeds[b, :S - 3] if q0 <= s < q0 + Lq]
+        assert inside
+        seeds[b, -1] = inside[0]          # a later slot repeats a window seed
+        seeds[b, -2] = -1
+        seeds[b, -3] = Lk + 5
+    _check(q, kc, vc, km, vm, seeds, q0, Lq)
+
+
+def test_packed_window_rows_match_square_rows():
+    # the packed kernel's rows agree with the same rows of the square launch up to rounding, and
+    # back-to-back calls give identical bits
+    B, Hq, Hkv, Lk, S = 2, 8, 2, 1100, 20
+    q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, S, 300, 200, "bf16", 7, 10)
+    dq, dk, dv, dkm, dvm = (H.to_dev(x, "bf16") for x in (q, kc, vc, km, vm))
+    ds = H.to_dev(seeds, "i32")
+    full, full_lse = api.cover_attn_fwd(dq, dk, dv, dkm, dvm, ds)
+    for q0, Lq in ((1099, 1), (300, 32), (1068, 32), (0, 64)):
+        win, win_lse = api.cover_attn_fwd_prefix(dq[:, :, q0:q0 + Lq].contiguous(), dk, dv, dkm, dvm, ds, q0=q0)
+        again, again_lse = api.cover_attn_fwd_prefix(dq[:, :, q0:q0 + Lq].contiguous(), dk, dv, dkm, dvm, ds, q0=q0)
+        torch.cuda.synchronize()
+        d = (win.float() - full[:, :, q0:q0 + Lq].float()).abs()
+        assert d.max().item() <= H.TOL_BF16_MAX and d.mean().item() <= H.TOL_BF16_MEAN, (q0, Lq)
+        assert (win_lse - full_lse[:, :, q0:q0 + Lq]).abs().max().item() <= H.TOL_LSE, (q0, Lq)
+        assert torch.equal(win, again) and torch.equal(win_lse, again_lse), (q0, Lq)
+    assert api.cover_device_status() == 0
