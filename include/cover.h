@@ -101,12 +101,15 @@ int cover_attn_fwd_f32(const float* q, const float* k_cached, const float* v_cac
  * With Lq = Lk and q0 = 0 this is cover_attn_fwd. Types, layouts, ownership
  * and errors as cover_attn_fwd / cover_attn_fwd_f32, plus
  * COVER_ERR_INVALID_ARG for Lq < 1, Lk < 1, q0 < 0 or q0 + Lq > Lk.
- * The bf16 call runs a short window of grouped-query heads (G = Hq / Hkv >= 2,
- * Lq <= 256, G * Lq <= 256, Lk <= 8192) on a kernel of its own: the G query
+ * The bf16 call may run a window of grouped-query heads (G = Hq / Hkv >= 2,
+ * Lq <= 256, G * Lq <= 1024, Lk <= 8192) on a kernel of its own: the G query
  * heads of a KV head packed into common Q tiles, the keys split over a cluster
- * of up to 8 CTAs that combine their partial softmax states. Its rows agree
- * with the square kernel's up to rounding (not bit for bit); any other window
- * runs on the square kernel, whose window rows equal the square launch's.
+ * of up to 8 CTAs that combine their partial softmax states. It does so where
+ * a launch-time model (the clusters that fit on the GPU at once, the KV steps
+ * of each kernel's longest chain) predicts it to be faster than the square
+ * kernel. Its rows agree with the square kernel's up to rounding (not bit for
+ * bit); any other window runs on the square kernel, whose window rows equal
+ * the square launch's.
  */
 int cover_attn_fwd_prefix(const void* q, const void* k_cached, const void* v_cached,
                           const void* k_seedmask, const void* v_seedmask,

@@ -38,9 +38,9 @@ int cover_debug_umma_tile(const void* a, const void* b, const void* p, const voi
 int cover_debug_wait_timeout(int limit_us, void* stream);
 
 /*
- * cover_attn_fwd_prefix (with Lq == Lk and q0 == 0: cover_attn_fwd) with a
- * fault planted on purpose, to drive the bf16 attention kernel's own abort
- * path: CTA `fault_cta` of the persistent grid leaves out the K tile load of
+ * The square bf16 attention kernel (the one cover_attn_fwd runs; windows as in
+ * cover_attn_fwd_prefix) with a fault planted on purpose, to drive its own
+ * abort path: CTA `fault_cta` of the persistent grid leaves out the K tile load of
  * its KV ring entry `fault_entry` (entries count the CTA's KV tiles over all
  * of its work units, from 0), and every bounded wait of the launch gives up
  * after `limit_us` microseconds (1 .. 2000000) instead of one second.
@@ -49,7 +49,8 @@ int cover_debug_wait_timeout(int limit_us, void* stream);
  * role of that CTA leaves its loop, lets the copies and tensor-core products
  * it already issued complete, frees its tensor memory and returns; the other
  * CTAs finish their units normally. The failed CTA's output rows are
- * unspecified. An entry the CTA never reaches plants nothing.
+ * unspecified. An entry the CTA never reaches plants nothing, and
+ * fault_cta = -1 gives a clean launch of the same kernel.
  * Arguments, layouts and errors otherwise as cover_attn_fwd_prefix (bf16).
  */
 int cover_debug_attn_fault(const void* q, const void* k_cached, const void* v_cached,
@@ -60,13 +61,30 @@ int cover_debug_attn_fault(const void* q, const void* k_cached, const void* v_ca
                            void* stream);
 
 /*
+ * cover_attn_fwd_prefix (bf16) on the packed grouped-query window kernel,
+ * whichever kernel the call itself would pick: cover_attn_fwd_prefix runs a
+ * window of grouped-query heads on the packed kernel only where a launch-time
+ * model predicts it to be faster than the square kernel. For tests of the
+ * packed kernel on every shape it supports. Arguments, layouts and errors as
+ * cover_attn_fwd_prefix, plus COVER_ERR_UNSUPPORTED where the packed kernel
+ * does not apply: Hq / Hkv < 2, Lq > 256, (Hq / Hkv) Lq > 1024, Lk > 8192,
+ * Lq == Lk with q0 == 0, or a cluster of its CTAs that cannot be resident.
+ */
+int cover_debug_attn_prefix_packed(const void* q, const void* k_cached, const void* v_cached,
+                                   const void* k_seedmask, const void* v_seedmask,
+                                   const int32_t* seed_idx, int n_seeds,
+                                   int B, int Hq, int Hkv, int Lq, int Lk, int q0, int D,
+                                   void* out, float* lse, void* stream);
+
+/*
  * Like cover_device_status, and also returns where the failure came from:
  * synchronises `stream`, copies the current device's status block to the
  * host array detail[3] = {status code, site id, linear block id} (all 0 when
  * nothing failed), clears it, and returns COVER_OK (COVER_ERR_CUDA if a CUDA
  * call fails). Site ids of the bf16 attention kernel: 10 TMA thread, 20 MMA
  * thread, 30 / 31 softmax warpgroup of Q tile 0 / 1, 40 routing warp,
- * 50 / 51 seed-score warp.
+ * 50 / 51 seed-score warp; of the packed window kernel: 60 TMA / MMA thread,
+ * 61 softmax warps, 62 combine (receive barrier), 63 copy issue.
  */
 int cover_debug_status_detail(int32_t* detail, void* stream);
 

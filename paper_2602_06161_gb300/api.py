@@ -440,6 +440,14 @@ def cover_debug_wait_timeout(limit_us: int, *, stream=None) -> None:
     _lib.check("cover_debug_wait_timeout", _lib.load().cover_debug_wait_timeout(int(limit_us), _stream(stream)))
 
 
+def cover_debug_attn_prefix_packed(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, seed_idx=None, *,
+                                   q0: int, out=None, lse=None, want_lse=True, stream=None):
+    """The prefix-window attention (bf16) on the packed grouped-query window kernel, whichever kernel
+    cover_attn_fwd_prefix would pick for the shape."""
+    return _attn_prefix("cover_debug_attn_prefix_packed", torch.bfloat16, q, k_cached, v_cached, k_seedmask,
+                        v_seedmask, seed_idx, q0, out, lse, want_lse, stream)
+
+
 def cover_debug_attn_fault(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, seed_idx=None, *, q0: int = 0,
                            fault_cta: int, fault_entry: int, limit_us: int, out=None, lse=None, stream=None):
     """Self-test: the bf16 attention (window form) with CTA fault_cta leaving out one K tile load and every

@@ -555,7 +555,86 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-bool window_gqa_applies(const AttnArgs& a) {
+namespace {
+
+// Launch set-up of one context: the kernel's shared-memory limit set, the SM count, and how many
+// clusters of each size (1 .. kMaxSplit CTAs of this kernel) can be resident at once.
+struct WinSetup {
+  int n_sm;
+  int max_clusters[kMaxSplit + 1];
+};
+
+// Shape of a packed launch: T KV tiles per CTA, nsplit CTAs per cluster, n_qt Q tiles per KV head.
+struct WinShape {
+  int G, nkv, T, nsplit, n_qt;
+  long long clusters;
+};
+
+WinShape win_shape(const AttnArgs& a) {
+  WinShape w;
+  w.G = a.Hq / a.Hkv;
+  w.nkv = (a.L + kBN - 1) / kBN;
+  w.T = (w.nkv + kMaxSplit - 1) / kMaxSplit;
+  w.nsplit = (w.nkv + w.T - 1) / w.T;   // every split has at least one KV tile
+  w.n_qt = (w.G * a.Lq + kBM - 1) / kBM;
+  w.clusters = static_cast<long long>(w.n_qt) * a.Hkv * a.B;
+  return w;
+}
+
+int win_setup(WinSetup* out, size_t smem) {
+  static ContextCache<WinSetup> setup;
+  return setup.get(out, [&](WinSetup& v) {
+    int dev = 0;
+    if (cudaFuncSetAttribute(attn_window_gqa_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem)) != cudaSuccess ||
+        cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&v.n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return -3;
+    v.max_clusters[0] = 0;
+    for (int cs = 1; cs <= kMaxSplit; ++cs) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(static_cast<unsigned>(cs));
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = smem;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = static_cast<unsigned>(cs);
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, attn_window_gqa_kernel, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+      }
+      v.max_clusters[cs] = n;
+    }
+    return 0;
+  });
+}
+
+// Predicted microseconds of one call on each kernel, fitted to calls measured back to back on
+// GB300 (Dream-shaped windows of 16 to 128 rows over 1024 keys, batches of 1 to 8, memories of
+// 2048 to 8192 keys; within 15 % on every shape measured): a packed CTA takes about 7 us plus
+// 1.5 us per KV step, and the clusters beyond those resident at once run in further waves; the
+// square kernel's window path takes about 5 us plus 1.7 us per KV step of one softmax warpgroup
+// for each round of its persistent grid.
+double packed_us(const WinShape& w, const WinSetup& su) {
+  const long long waves = (w.clusters + su.max_clusters[w.nsplit] - 1) / su.max_clusters[w.nsplit];
+  return static_cast<double>(waves) * (7.0 + 1.5 * w.T);
+}
+
+double square_us(const AttnArgs& a, const WinShape& w, const WinSetup& su) {
+  const long long units = static_cast<long long>((a.Lq + 255) / 256) * a.Hq * a.B;
+  const long long rounds = (units + su.n_sm - 1) / su.n_sm;
+  // a window of at most 128 rows with an even number of KV tiles splits each unit's keys over
+  // the two softmax warpgroups
+  const int steps = (a.Lq <= kBM && w.nkv % 2 == 0) ? w.nkv / 2 : w.nkv;
+  return 5.0 + static_cast<double>(rounds) * steps * 1.7;
+}
+
+bool packed_supported(const AttnArgs& a) {
   const bool window = a.Lq != a.L || a.q0 != 0;
   const int G = a.Hkv > 0 ? a.Hq / a.Hkv : 0;
   const int nkv = (a.L + kBN - 1) / kBN;
@@ -564,13 +643,18 @@ bool window_gqa_applies(const AttnArgs& a) {
          static_cast<long long>(a.B) * a.Hq * a.Lq + kBM < 0x7fffffffLL;
 }
 
-int launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream) {
-  const int G = a.Hq / a.Hkv;
-  const int nkv = (a.L + kBN - 1) / kBN;
-  const int T = (nkv + kMaxSplit - 1) / kMaxSplit;    // KV steps per CTA
-  const int nsplit = (nkv + T - 1) / T;               // every split has at least one KV tile
-  const int n_qt = (G * a.Lq + kBM - 1) / kBM;
-  const long long grid = static_cast<long long>(nsplit) * n_qt * a.Hkv * a.B;
+}  // namespace
+
+int try_launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream, bool force) {
+  if (!packed_supported(a)) return kWindowGqaNotTaken;
+  const size_t smem = sizeof(WinSmem) + 1024;
+  WinSetup su;
+  const int rc = win_setup(&su, smem);
+  if (rc != 0) return rc;
+  const WinShape w = win_shape(a);
+  if (su.max_clusters[w.nsplit] < 1) return kWindowGqaNotTaken;   // such a cluster cannot be resident
+  if (!force && packed_us(w, su) >= square_us(a, w, su)) return kWindowGqaNotTaken;
+  const long long grid = w.clusters * w.nsplit;
   if (grid > 0x7fffffffLL) return -2;
   CUtensorMap tq, tk, tv;
   // q as one [B * Hq * Lq, D] matrix; K', V' as [B, Hkv, Lk, D]
@@ -578,14 +662,6 @@ int launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream) 
       !make_bf16_map_4d(&tk, a.k_cached, kD, a.L, a.Hkv, a.B, kBN) ||
       !make_bf16_map_4d(&tv, a.v_cached, kD, a.L, a.Hkv, a.B, kBN))
     return -3;
-  const size_t smem = sizeof(WinSmem) + 1024;
-  static ContextCache<int> setup;
-  int unused = 0;
-  const int rc = setup.get(&unused, [&](int&) {
-    return cudaFuncSetAttribute(attn_window_gqa_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                static_cast<int>(smem)) == cudaSuccess ? 0 : -3;
-  });
-  if (rc != 0) return rc;
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kD));
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(grid));
@@ -594,7 +670,7 @@ int launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream) 
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = static_cast<unsigned>(nsplit);
+  attr[0].val.clusterDim.x = static_cast<unsigned>(w.nsplit);
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   // programmatic dependent launch: the prologue overlaps the previous kernel's tail
@@ -605,8 +681,8 @@ int launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream) 
   const cudaError_t e = cudaLaunchKernelEx(
       &cfg, attn_window_gqa_kernel, tq, tk, tv, static_cast<const __nv_bfloat16*>(a.q),
       static_cast<const __nv_bfloat16*>(a.k_seedmask), static_cast<const __nv_bfloat16*>(a.v_seedmask), a.seed_idx,
-      a.n_seeds, a.Hq, a.Hkv, G, a.Lq, a.L, a.q0, n_qt, nsplit, T, scale_log2, static_cast<__nv_bfloat16*>(a.out),
-      a.lse, status, kWaitLimitNs);
+      a.n_seeds, a.Hq, a.Hkv, w.G, a.Lq, a.L, a.q0, w.n_qt, w.nsplit, w.T, scale_log2,
+      static_cast<__nv_bfloat16*>(a.out), a.lse, status, kWaitLimitNs);
   return e == cudaSuccess && cudaGetLastError() == cudaSuccess ? 0 : -3;
 }
 

@@ -96,7 +96,8 @@ int cover_attn_fwd_prefix(const void* q, const void* k_cached, const void* v_cac
   if (st == nullptr) return COVER_ERR_CUDA;
   cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
                     Lq, q0};
-  if (cover::window_gqa_applies(a)) return cover::launch_attn_window_gqa(a, st, static_cast<cudaStream_t>(stream));
+  const int pk = cover::try_launch_attn_window_gqa(a, st, static_cast<cudaStream_t>(stream), false);
+  if (pk != cover::kWindowGqaNotTaken) return pk;
   return cover::launch_attn_bf16_sm103(a, st, static_cast<cudaStream_t>(stream));
 }
 
@@ -345,6 +346,23 @@ int cover_debug_umma_tile(const void* a, const void* b, const void* p, const voi
   int* st = status_block();
   if (st == nullptr) return COVER_ERR_CUDA;
   return cover::launch_umma_tile(a, b, p, v, c1, c2, st, static_cast<cudaStream_t>(stream));
+}
+
+int cover_debug_attn_prefix_packed(const void* q, const void* k_cached, const void* v_cached, const void* k_seedmask,
+                                   const void* v_seedmask, const int32_t* seed_idx, int n_seeds, int B, int Hq,
+                                   int Hkv, int Lq, int Lk, int q0, int D, void* out, float* lse, void* stream) {
+  int rc = check_window(Lq, Lk, q0);
+  if (rc != COVER_OK) return rc;
+  rc = check_attn_args(q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
+                       16);
+  if (rc != COVER_OK) return rc;
+  if (D != 128) return COVER_ERR_UNSUPPORTED;
+  int* st = status_block();
+  if (st == nullptr) return COVER_ERR_CUDA;
+  cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
+                    Lq, q0};
+  rc = cover::try_launch_attn_window_gqa(a, st, static_cast<cudaStream_t>(stream), true);
+  return rc == cover::kWindowGqaNotTaken ? COVER_ERR_UNSUPPORTED : rc;
 }
 
 int cover_debug_attn_fault(const void* q, const void* k_cached, const void* v_cached, const void* k_seedmask,

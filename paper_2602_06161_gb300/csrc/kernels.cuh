@@ -31,14 +31,16 @@ struct AttnArgs {
 int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream);
 
 // Prefix-cache windows of grouped-query heads (attn_window_gqa.cu): the G = Hq / Hkv query heads
-// of a KV head packed into common Q tiles, the keys split over a cluster of up to 8 CTAs. Taken
-// for a window (Lq != L or q0 != 0) with G >= 2, Lq <= kMaxWindowGqaRows,
+// of a KV head packed into common Q tiles, the keys split over a cluster of up to 8 CTAs.
+// Supported for a window (Lq != L or q0 != 0) with G >= 2, Lq <= kMaxWindowGqaRows,
 // G * Lq <= kMaxWindowGqaPacked and at most 8 * kMaxWindowGqaSteps KV tiles of 128 keys.
+// try_launch_attn_window_gqa launches it where it is supported and (unless `force`) predicted to
+// be faster than the square kernel's window path, and returns kWindowGqaNotTaken otherwise.
 constexpr int kMaxWindowGqaRows = 256;
-constexpr int kMaxWindowGqaPacked = 256;
+constexpr int kMaxWindowGqaPacked = 1024;
 constexpr int kMaxWindowGqaSteps = 8;
-bool window_gqa_applies(const AttnArgs& a);
-int launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream);
+constexpr int kWindowGqaNotTaken = 1;
+int try_launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream, bool force);
 int launch_attn_f32(const AttnArgs& a, int* status, cudaStream_t stream);
 
 int launch_seed_route(const int32_t* seed_idx, int n_seeds, int B, int L, int32_t* slot_out, uint32_t* bitmap_out,

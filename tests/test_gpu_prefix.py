@@ -75,16 +75,17 @@ def test_window_f32(D, Lk, Lq, q0):
 def test_window_rows_equal_square_rows_bit_exactly():
     # a query row's arithmetic does not depend on where its tile starts: the window rows
     # are bit-identical to the same rows of the square launch (an odd number of KV tiles,
-    # so the square launch does not split any unit's keys over two CTAs). Windows of at most
-    # 256 packed rows (G * Lq) go to the packed grouped-query kernel instead, whose rows agree
-    # with the square launch up to rounding (test_gpu_window_gqa.py)
+    # so the square launch does not split any unit's keys over two CTAs). The windows run on the
+    # square kernel through the fault entry with no planted load: the prefix call itself may take
+    # the packed grouped-query kernel, whose rows agree up to rounding (test_gpu_window_gqa.py)
     B, Hq, Hkv, Lk, S = 2, 4, 2, 1100, 20
     q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, S, 300, 200, "bf16", 7, 10)
     dq, dk, dv, dkm, dvm = (H.to_dev(x, "bf16") for x in (q, kc, vc, km, vm))
     ds = H.to_dev(seeds, "i32")
     full, full_lse = api.cover_attn_fwd(dq, dk, dv, dkm, dvm, ds)
-    for q0, Lq in ((300, 200), (0, 1100), (130, 257), (971, 129)):
-        win, win_lse = api.cover_attn_fwd_prefix(dq[:, :, q0:q0 + Lq].contiguous(), dk, dv, dkm, dvm, ds, q0=q0)
+    for q0, Lq in ((300, 200), (0, 1100), (1099, 1), (130, 257)):
+        win, win_lse = api.cover_debug_attn_fault(dq[:, :, q0:q0 + Lq].contiguous(), dk, dv, dkm, dvm, ds, q0=q0,
+                                                  fault_cta=-1, fault_entry=-1, limit_us=1000000)
         torch.cuda.synchronize()
         assert torch.equal(win, full[:, :, q0:q0 + Lq]), (q0, Lq)
         assert torch.equal(win_lse, full_lse[:, :, q0:q0 + Lq]), (q0, Lq)

@@ -1,5 +1,9 @@
 """GPU parity of the packed grouped-query window kernel (the prefix-cache window of Section 6.6
-for G = Hq / Hkv >= 2 and G * Lq <= 256 packed rows) against the fp64 oracle.
+for G = Hq / Hkv >= 2) against the fp64 oracle, and the choice between it and the square kernel.
+
+cover_attn_fwd_prefix runs a window of grouped-query heads on the packed kernel where a launch-time
+model predicts it to be faster; cover_debug_attn_prefix_packed runs the packed kernel on every
+shape it supports, which the parity cases below use.
 
 The kernel packs a KV head's G query heads into common 128-row Q tiles and splits the keys over
 the CTAs of a cluster (T = ceil(nkv / 8) KV tiles per CTA, nsplit = ceil(nkv / T) CTAs), which
@@ -13,16 +17,25 @@ import pytest
 import torch
 
 import oracle
-from paper_2602_06161_gb300 import api
+from paper_2602_06161_gb300 import CoverError, api
 from paper_2602_06161_gb300 import workloads as W
 from tests import _gpu as H
-from tests.test_gpu_prefix import _case, run_window
+from tests.test_gpu_prefix import _case
 
 pytestmark = pytest.mark.gpu
 
 
+def _packed(q, kc, vc, km, vm, seeds, q0, Lq):
+    out, lse = api.cover_debug_attn_prefix_packed(
+        H.to_dev(np.ascontiguousarray(q[:, :, q0:q0 + Lq]), "bf16"), H.to_dev(kc, "bf16"), H.to_dev(vc, "bf16"),
+        H.to_dev(km, "bf16"), H.to_dev(vm, "bf16"), H.to_dev(seeds, "i32"), q0=q0)
+    torch.cuda.synchronize()
+    assert api.cover_device_status() == 0
+    return out.float().cpu().numpy(), lse.cpu().numpy()
+
+
 def _check(q, kc, vc, km, vm, seeds, q0, Lq):
-    out, lse = run_window(q, kc, vc, km, vm, seeds, q0, Lq, "bf16")
+    out, lse = _packed(q, kc, vc, km, vm, seeds, q0, Lq)
     f = W.bf16_bits_to_f64
     ref, ref_lse = oracle.override_attention_window(f(q[:, :, q0:q0 + Lq]), f(kc), f(vc), f(km), f(vm),
                                                     seeds if seeds.shape[1] else None, q0)
@@ -41,6 +54,8 @@ def _check(q, kc, vc, km, vm, seeds, q0, Lq):
     (2, 9, 3, 333, 37, 100, 7, 3),         # 111 packed rows: the last warp's rows end mid-warp
     (1, 16, 2, 640, 16, 624, 5, 2),        # G = 8: one full Q tile
     (3, 10, 5, 90, 3, 40, 4, 2),           # one ragged KV tile: a cluster of one CTA
+    (1, 28, 4, 1024, 128, 896, 32, 20),    # 896 packed rows: 7 Q tiles per KV head
+    (2, 28, 4, 2048, 64, 1984, 24, 10),    # 16 KV tiles: 8 CTAs of 2 steps, 4 Q tiles
 ])
 def test_packed_window_matches_oracle(B, Hq, Hkv, Lk, Lq, q0, S, inside):
     q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, S, q0, Lq, "bf16", 3 * Lk + Lq, inside)
@@ -80,11 +95,49 @@ def test_packed_window_rows_match_square_rows():
     ds = H.to_dev(seeds, "i32")
     full, full_lse = api.cover_attn_fwd(dq, dk, dv, dkm, dvm, ds)
     for q0, Lq in ((1099, 1), (300, 32), (1068, 32), (0, 64)):
-        win, win_lse = api.cover_attn_fwd_prefix(dq[:, :, q0:q0 + Lq].contiguous(), dk, dv, dkm, dvm, ds, q0=q0)
-        again, again_lse = api.cover_attn_fwd_prefix(dq[:, :, q0:q0 + Lq].contiguous(), dk, dv, dkm, dvm, ds, q0=q0)
+        qw = dq[:, :, q0:q0 + Lq].contiguous()
+        win, win_lse = api.cover_debug_attn_prefix_packed(qw, dk, dv, dkm, dvm, ds, q0=q0)
+        again, again_lse = api.cover_debug_attn_prefix_packed(qw, dk, dv, dkm, dvm, ds, q0=q0)
         torch.cuda.synchronize()
         d = (win.float() - full[:, :, q0:q0 + Lq].float()).abs()
         assert d.max().item() <= H.TOL_BF16_MAX and d.mean().item() <= H.TOL_BF16_MEAN, (q0, Lq)
         assert (win_lse - full_lse[:, :, q0:q0 + Lq]).abs().max().item() <= H.TOL_LSE, (q0, Lq)
         assert torch.equal(win, again) and torch.equal(win_lse, again_lse), (q0, Lq)
     assert api.cover_device_status() == 0
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,Lk,Lq,packed", [
+    (1, 28, 4, 1024, 32, True),     # Dream active block: 8 clusters of 8 one-step CTAs
+    (1, 32, 8, 8192, 32, True),     # long memory: 8 steps per packed CTA against 32 per warpgroup
+    (3, 10, 5, 90, 3, False),       # one KV tile: the square kernel's short chain wins
+    (8, 32, 8, 2048, 64, False),    # 128 clusters: many waves of packed CTAs
+])
+def test_prefix_call_picks_the_predicted_kernel(B, Hq, Hkv, Lk, Lq, packed):
+    # the call's result equals, bit for bit, the kernel the launch-time model picks for the shape
+    q0 = Lk - Lq
+    q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, 6, q0, Lq, "bf16", 5 + Lk, 2)
+    dev = [H.to_dev(np.ascontiguousarray(q[:, :, q0:]), "bf16"), H.to_dev(kc, "bf16"), H.to_dev(vc, "bf16"),
+           H.to_dev(km, "bf16"), H.to_dev(vm, "bf16"), H.to_dev(seeds, "i32")]
+    prod, prod_lse = api.cover_attn_fwd_prefix(*dev, q0=q0)
+    pk, pk_lse = api.cover_debug_attn_prefix_packed(*dev, q0=q0)
+    sq, sq_lse = api.cover_debug_attn_fault(*dev, q0=q0, fault_cta=-1, fault_entry=-1, limit_us=1000000)
+    torch.cuda.synchronize()
+    assert api.cover_device_status() == 0
+    ref = (pk, pk_lse) if packed else (sq, sq_lse)
+    assert torch.equal(prod, ref[0]) and torch.equal(prod_lse, ref[1])
+    assert (pk.float() - sq.float()).abs().max().item() <= H.TOL_BF16_MAX
+
+
+def test_packed_entry_refuses_what_the_packed_kernel_does_not_run():
+    q, kc, vc, km, vm, seeds = _case(1, 4, 4, 256, 128, 4, 192, 64, "bf16", 9, 2)
+    dev = [H.to_dev(kc, "bf16"), H.to_dev(vc, "bf16"), H.to_dev(km, "bf16"), H.to_dev(vm, "bf16"),
+           H.to_dev(seeds, "i32")]
+    with pytest.raises(CoverError) as e:   # G = 1: no query heads to pack
+        api.cover_debug_attn_prefix_packed(H.to_dev(np.ascontiguousarray(q[:, :, 192:]), "bf16"), *dev, q0=192)
+    assert e.value.code == -2
+    q, kc, vc, km, vm, seeds = _case(1, 4, 2, 256, 128, 4, 0, 256, "bf16", 9, 2)
+    with pytest.raises(CoverError) as e:   # the square call
+        api.cover_debug_attn_prefix_packed(H.to_dev(q, "bf16"), H.to_dev(kc, "bf16"), H.to_dev(vc, "bf16"),
+                                           H.to_dev(km, "bf16"), H.to_dev(vm, "bf16"), H.to_dev(seeds, "i32"),
+                                           q0=0)
+    assert e.value.code == -2
