@@ -59,7 +59,7 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-secondary", action="store_true")
-    ap.add_argument("--only", choices=["attn", "prefix", "score", "decide", "mass", "kv"], default=None,
+    ap.add_argument("--only", choices=["attn", "prefix", "prefix_gqa", "score", "decide", "mass", "kv"], default=None,
                     help="time one kernel alone on the workload (for profiler captures)")
     return ap.parse_args()
 
@@ -848,6 +848,18 @@ def run_only(args):
         qw = q[:, :, q0:].contiguous()
         out, lse = torch.empty_like(qw), torch.empty((wl.B, wl.Hq, 64), device="cuda")
         fn = lambda: api.cover_attn_fwd_prefix(qw, kc, vc, km, vm, seeds, q0=q0, out=out, lse=lse)  # noqa: E731
+    elif args.only == "prefix_gqa":
+        # the Dream-shaped 32-row block over its 1024-position memory (28 query heads on 4 KV heads),
+        # which takes the packed grouped-query window kernel
+        gw = W.WORKLOADS["dream_gqa_l1024"]
+        ai = gw.attn_inputs()
+        q, kc, vc = bf16_dev(ai.q, torch), bf16_dev(ai.k_cached, torch), bf16_dev(ai.v_cached, torch)
+        km, vm = bf16_dev(ai.k_seedmask, torch), bf16_dev(ai.v_seedmask, torch)
+        seeds = torch.from_numpy(ai.seed_idx).cuda()
+        q0 = gw.L - 32
+        qw = q[:, :, q0:].contiguous()
+        out, lse = torch.empty_like(qw), torch.empty((gw.B, gw.Hq, 32), device="cuda")
+        fn = lambda: api.cover_attn_fwd_prefix(qw, kc, vc, km, vm, seeds, q0=q0, out=out, lse=lse)  # noqa: E731
     elif args.only == "score":
         si = wl.score_inputs()
         logits = bf16_dev(si.logits, torch)
@@ -891,7 +903,8 @@ def run_only(args):
     status = api.cover_device_status()
     if status != 0:
         raise RuntimeError(api.cover_status_str(status))
-    return {"only": args.only, "workload": WORKLOAD, "ms_per_launch": round(a.elapsed_time(b) / args.steps, 4),
+    return {"only": args.only, "workload": "dream_gqa_l1024" if args.only == "prefix_gqa" else WORKLOAD,
+            "ms_per_launch": round(a.elapsed_time(b) / args.steps, 4),
             "kernel_source_hash": kernel_source_hash()}
 
 
