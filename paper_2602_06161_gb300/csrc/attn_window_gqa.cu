@@ -40,6 +40,7 @@
 #include <cuda_fp16.h>
 #include <math.h>
 
+#include "cluster.cuh"
 #include "context.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
