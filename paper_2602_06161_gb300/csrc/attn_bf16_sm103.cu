@@ -68,6 +68,10 @@ constexpr int kTmaWarp = 9;
 constexpr int kRouteWarp = 10;
 constexpr int kSeedWarp = 11;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+// A seed row's self term e^{s_self} is merged at the row's reference m as (O + p v) / (l + p),
+// p = 2^(s_self - m) (equal to rescaling all three to max(m, s_self)), while s_self <= m + 64
+// keeps p and O + p v far inside fp32; above that (m, l, O) is rescaled to s_self instead.
+constexpr float kSelfInPlace = 64.0f;      // log2 units
 constexpr int kVStageRows = 32;            // masked value rows of a unit staged in shared memory
 constexpr int kNotStaged = 255;
 
@@ -879,22 +883,40 @@ __global__ void __launch_bounds__(kThreads, 1)
             const size_t mrow = ((static_cast<size_t>(w.b) * Hkv + ug.group.div(static_cast<uint32_t>(w.hq))) * n_seeds + my_slot) * kD;
             const uint4* vmv = (vi != kNotStaged ? reinterpret_cast<const uint4*>(sm.vstage[sb][vi])
                                                  : reinterpret_cast<const uint4*>(v_seedmask + mrow)) + cb / 8;
-            const float m2 = fmaxf(m, s_self);
-            const float a = (m == -INFINITY) ? 0.0f : ex2_approx(m - m2);
-            const float pself = ex2_approx(s_self - m2);
-            l = l * a + pself;
+            if (m != -INFINITY && s_self <= m + kSelfInPlace) {
+              // (O + p v) / (l + p) with p = 2^(s_self - m): one multiply-add per element
+              const float pself = ex2_approx(s_self - m);
+              l += pself;
 #pragma unroll
-            for (int ch = 0; ch < 8; ++ch) {
-              const uint4 vv = vmv[ch];
-              const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
+              for (int ch = 0; ch < 8; ++ch) {
+                const uint4 vv = vmv[ch];
+                const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
 #pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const float2 vf = __bfloat1622float2(vp[e]);
-                oh[ch * 8 + 2 * e] = oh[ch * 8 + 2 * e] * a + pself * vf.x;
-                oh[ch * 8 + 2 * e + 1] = oh[ch * 8 + 2 * e + 1] * a + pself * vf.y;
+                for (int e = 0; e < 4; ++e) {
+                  const float2 vf = __bfloat1622float2(vp[e]);
+                  oh[ch * 8 + 2 * e] = fmaf(pself, vf.x, oh[ch * 8 + 2 * e]);
+                  oh[ch * 8 + 2 * e + 1] = fmaf(pself, vf.y, oh[ch * 8 + 2 * e + 1]);
+                }
               }
+            } else {
+              // a self term far above the row's other scores: rescale (m, l, O) to it
+              const float m2 = fmaxf(m, s_self);
+              const float a = (m == -INFINITY) ? 0.0f : ex2_approx(m - m2);
+              const float pself = ex2_approx(s_self - m2);
+              l = l * a + pself;
+#pragma unroll
+              for (int ch = 0; ch < 8; ++ch) {
+                const uint4 vv = vmv[ch];
+                const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const float2 vf = __bfloat1622float2(vp[e]);
+                  oh[ch * 8 + 2 * e] = oh[ch * 8 + 2 * e] * a + pself * vf.x;
+                  oh[ch * 8 + 2 * e + 1] = oh[ch * 8 + 2 * e + 1] * a + pself * vf.y;
+                }
+              }
+              m = m2;
             }
-            m = m2;
           }
           const int sig = (g0 + nkv - 1) & 1;
           uint8_t* stage = sm.k[sig] + (warp & 3) * (2 * 4096) + qt * 4096;
@@ -941,22 +963,40 @@ __global__ void __launch_bounds__(kThreads, 1)
           // generic loads: shared memory when warp 11 staged the row, else global memory
           const uint4* vmv = vi != kNotStaged ? reinterpret_cast<const uint4*>(sm.vstage[sb][vi])
                                               : reinterpret_cast<const uint4*>(v_seedmask + mrow);
-          const float m2 = fmaxf(m_run, s_self);
-          const float a = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m2);
-          const float pself = ex2_approx(s_self - m2);
-          l_run = l_run * a + pself;
+          if (m_run != -INFINITY && s_self <= m_run + kSelfInPlace) {
+            // (O + p v) / (l + p) with p = 2^(s_self - m): one multiply-add per element
+            const float pself = ex2_approx(s_self - m_run);
+            l_run += pself;
 #pragma unroll
-          for (int ch = 0; ch < 16; ++ch) {
-            const uint4 vv = vmv[ch];
-            const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
+            for (int ch = 0; ch < 16; ++ch) {
+              const uint4 vv = vmv[ch];
+              const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 vf = __bfloat1622float2(vp[e]);
-              o[ch * 8 + 2 * e] = o[ch * 8 + 2 * e] * a + pself * vf.x;
-              o[ch * 8 + 2 * e + 1] = o[ch * 8 + 2 * e + 1] * a + pself * vf.y;
+              for (int e = 0; e < 4; ++e) {
+                const float2 vf = __bfloat1622float2(vp[e]);
+                o[ch * 8 + 2 * e] = fmaf(pself, vf.x, o[ch * 8 + 2 * e]);
+                o[ch * 8 + 2 * e + 1] = fmaf(pself, vf.y, o[ch * 8 + 2 * e + 1]);
+              }
             }
+          } else {
+            // a self term far above the row's other scores: rescale (m, l, O) to it
+            const float m2 = fmaxf(m_run, s_self);
+            const float a = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m2);
+            const float pself = ex2_approx(s_self - m2);
+            l_run = l_run * a + pself;
+#pragma unroll
+            for (int ch = 0; ch < 16; ++ch) {
+              const uint4 vv = vmv[ch];
+              const __nv_bfloat162* vp = reinterpret_cast<const __nv_bfloat162*>(&vv);
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float2 vf = __bfloat1622float2(vp[e]);
+                o[ch * 8 + 2 * e] = o[ch * 8 + 2 * e] * a + pself * vf.x;
+                o[ch * 8 + 2 * e + 1] = o[ch * 8 + 2 * e + 1] * a + pself * vf.y;
+              }
+            }
+            m_run = m2;
           }
-          m_run = m2;
         }
         // Output: the warp's 32 rows x 128 columns are staged in the shared-memory stage of
         // the unit's last KV tile (K stage for Q tile 0, V stage for Q tile 1: both finished
