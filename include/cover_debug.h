@@ -65,16 +65,26 @@ int cover_debug_attn_fault(const void* q, const void* k_cached, const void* v_ca
  * whichever kernel the call itself would pick: cover_attn_fwd_prefix runs a
  * window of grouped-query heads on the packed kernel only where a launch-time
  * model predicts it to be faster than the square kernel. For tests of the
- * packed kernel on every shape it supports. Arguments, layouts and errors as
- * cover_attn_fwd_prefix, plus COVER_ERR_UNSUPPORTED where the packed kernel
- * does not apply: Hq / Hkv < 2, Lq > 256, (Hq / Hkv) Lq > 1024, Lk > 8192,
- * Lq == Lk with q0 == 0, or a cluster of its CTAs that cannot be resident.
+ * packed kernel on every shape it supports. With fault_cta >= 0 or
+ * limit_us > 0 it runs the kernel's self-test instance instead: CTA fault_cta
+ * (grid order: key split fastest, then Q tile, KV head, batch row) leaves out
+ * the K load of its first KV tile, and every bounded wait gives up after
+ * limit_us microseconds (1 .. 2000000; 0: one second). That CTA records
+ * COVER_ERR_DEVICE_TIMEOUT at site 60 or 61 (the first of its waits that
+ * depend on the tile to give up), every role leaves its loop, and the
+ * launch completes; the output rows of that CTA's cluster (its Q tile of its KV
+ * head) are unspecified, every other row is the clean result. fault_cta = -1
+ * with limit_us = 0 is the normal launch. Arguments, layouts and errors as
+ * cover_attn_fwd_prefix, plus COVER_ERR_INVALID_ARG for limit_us outside
+ * 0 .. 2000000, and COVER_ERR_UNSUPPORTED where the packed kernel does not
+ * apply: Hq / Hkv < 2, Lq > 256, (Hq / Hkv) Lq > 1024, Lk > 8192, Lq == Lk with
+ * q0 == 0, or a cluster of its CTAs that cannot be resident.
  */
 int cover_debug_attn_prefix_packed(const void* q, const void* k_cached, const void* v_cached,
                                    const void* k_seedmask, const void* v_seedmask,
                                    const int32_t* seed_idx, int n_seeds,
                                    int B, int Hq, int Hkv, int Lq, int Lk, int q0, int D,
-                                   void* out, float* lse, void* stream);
+                                   void* out, float* lse, int fault_cta, int limit_us, void* stream);
 
 /*
  * Like cover_device_status, and also returns where the failure came from:

@@ -39,7 +39,8 @@ _SIGNATURES = {
     "cover_status_str": (ctypes.c_char_p, [_I]),
     "cover_debug_umma_tile": (_I, [_P, _P, _P, _P, _P, _P, _P]),
     "cover_debug_wait_timeout": (_I, [_I, _P]),
-    "cover_debug_attn_prefix_packed": (_I, [_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
+    "cover_debug_attn_prefix_packed": (_I, [_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _P, _P, _I, _I,
+                                            _P]),
     "cover_debug_attn_fault": (_I, [_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _P, _P, _I, _I, _I,
                                     _P]),
     "cover_debug_status_detail": (_I, [_P, _P]),

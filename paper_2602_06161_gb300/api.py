@@ -441,11 +441,14 @@ def cover_debug_wait_timeout(limit_us: int, *, stream=None) -> None:
 
 
 def cover_debug_attn_prefix_packed(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, seed_idx=None, *,
-                                   q0: int, out=None, lse=None, want_lse=True, stream=None):
+                                   q0: int, fault_cta: int = -1, limit_us: int = 0, out=None, lse=None,
+                                   want_lse=True, stream=None):
     """The prefix-window attention (bf16) on the packed grouped-query window kernel, whichever kernel
-    cover_attn_fwd_prefix would pick for the shape."""
+    cover_attn_fwd_prefix would pick for the shape; fault_cta >= 0 or limit_us > 0 run its self-test
+    instance (CTA fault_cta leaves out its first K load, waits give up after limit_us)."""
     return _attn_prefix("cover_debug_attn_prefix_packed", torch.bfloat16, q, k_cached, v_cached, k_seedmask,
-                        v_seedmask, seed_idx, q0, out, lse, want_lse, stream)
+                        v_seedmask, seed_idx, q0, out, lse, want_lse, stream,
+                        extra=(int(fault_cta), int(limit_us)))
 
 
 def cover_debug_attn_fault(q, k_cached, v_cached, k_seedmask=None, v_seedmask=None, seed_idx=None, *, q0: int = 0,

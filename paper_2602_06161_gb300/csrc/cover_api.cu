@@ -350,7 +350,9 @@ int cover_debug_umma_tile(const void* a, const void* b, const void* p, const voi
 
 int cover_debug_attn_prefix_packed(const void* q, const void* k_cached, const void* v_cached, const void* k_seedmask,
                                    const void* v_seedmask, const int32_t* seed_idx, int n_seeds, int B, int Hq,
-                                   int Hkv, int Lq, int Lk, int q0, int D, void* out, float* lse, void* stream) {
+                                   int Hkv, int Lq, int Lk, int q0, int D, void* out, float* lse, int fault_cta,
+                                   int limit_us, void* stream) {
+  if (limit_us < 0 || limit_us > 2000000) return COVER_ERR_INVALID_ARG;
   int rc = check_window(Lq, Lk, q0);
   if (rc != COVER_OK) return rc;
   rc = check_attn_args(q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
@@ -361,6 +363,8 @@ int cover_debug_attn_prefix_packed(const void* q, const void* k_cached, const vo
   if (st == nullptr) return COVER_ERR_CUDA;
   cover::AttnArgs a{q, k_cached, v_cached, k_seedmask, v_seedmask, seed_idx, n_seeds, B, Hq, Hkv, Lk, D, out, lse,
                     Lq, q0};
+  a.fault_cta = fault_cta;
+  a.wait_ns = static_cast<uint64_t>(limit_us) * 1000ull;
   rc = cover::try_launch_attn_window_gqa(a, st, static_cast<cudaStream_t>(stream), true);
   return rc == cover::kWindowGqaNotTaken ? COVER_ERR_UNSUPPORTED : rc;
 }

@@ -36,6 +36,8 @@ int launch_attn_bf16_sm103(const AttnArgs& a, int* status, cudaStream_t stream);
 // G * Lq <= kMaxWindowGqaPacked and at most 8 * kMaxWindowGqaSteps KV tiles of 128 keys.
 // try_launch_attn_window_gqa launches it where it is supported and (unless `force`) predicted to
 // be faster than the square kernel's window path, and returns kWindowGqaNotTaken otherwise.
+// With `force`, a.fault_cta >= 0 or a.wait_ns > 0 select its self-test instance: CTA fault_cta
+// leaves out the K load of its first KV tile, every bounded wait gives up after wait_ns.
 constexpr int kMaxWindowGqaRows = 256;
 constexpr int kMaxWindowGqaPacked = 1024;
 constexpr int kMaxWindowGqaSteps = 8;

@@ -141,3 +141,39 @@ def test_packed_entry_refuses_what_the_packed_kernel_does_not_run():
                                            H.to_dev(km, "bf16"), H.to_dev(vm, "bf16"), H.to_dev(seeds, "i32"),
                                            q0=0)
     assert e.value.code == -2
+
+
+def test_packed_planted_missing_load_aborts_cleanly():
+    # The packed kernel's self-test instance: CTA 0 (key split 0 of Q tile 0 of KV head 0) leaves
+    # out its first K load and every wait gives up after 20 ms. Its waits for that tile time out
+    # (site 60 or 61 is recorded), every role leaves its loop, the cluster's copies and barriers still
+    # complete, and the launch returns well within a second. The rows CTA 0's cluster combines
+    # (packed rows 0..127 of KV head 0: query heads 0..3 of the Dream shape) are unspecified;
+    # every other row is bit-identical to a clean launch, and so is the next clean launch.
+    import time
+    B, Hq, Hkv, Lk, Lq, q0, S = 1, 28, 4, 1024, 32, 992, 32
+    q, kc, vc, km, vm, seeds = _case(B, Hq, Hkv, Lk, 128, S, q0, Lq, "bf16", 71, 6)
+    dev = [H.to_dev(np.ascontiguousarray(q[:, :, q0:]), "bf16"), H.to_dev(kc, "bf16"), H.to_dev(vc, "bf16"),
+           H.to_dev(km, "bf16"), H.to_dev(vm, "bf16"), H.to_dev(seeds, "i32")]
+    clean, clean_lse = api.cover_debug_attn_prefix_packed(*dev, q0=q0)
+    torch.cuda.synchronize()
+    assert api.cover_debug_status_detail() == (0, 0, 0)
+    out = torch.full_like(clean, float("nan"))
+    lse = torch.full_like(clean_lse, float("nan"))
+    t0 = time.perf_counter()
+    api.cover_debug_attn_prefix_packed(*dev, q0=q0, fault_cta=0, limit_us=20000, out=out, lse=lse)
+    code, site, block = api.cover_debug_status_detail()
+    elapsed = time.perf_counter() - t0
+    # the MMA thread's wait for the tile (60) or the softmax warps' wait for its product (61),
+    # whichever gives up first
+    assert code == -4 and site in (60, 61) and block == 0, (code, site, block)
+    assert elapsed < 0.5
+    assert api.cover_debug_status_detail() == (0, 0, 0)
+    G = Hq // Hkv
+    mine = torch.zeros((B, Hq, Lq), dtype=torch.bool, device="cuda")
+    mine.view(B, Hkv, G * Lq)[0, 0, :128] = True
+    assert torch.equal(out[~mine], clean[~mine]) and torch.equal(lse[~mine], clean_lse[~mine])
+    again, again_lse = api.cover_debug_attn_prefix_packed(*dev, q0=q0)
+    torch.cuda.synchronize()
+    assert api.cover_device_status() == 0
+    assert torch.equal(again, clean) and torch.equal(again_lse, clean_lse)
