@@ -107,6 +107,21 @@ __device__ __forceinline__ uint32_t part_off(int qr, int owner, int c) {
   return static_cast<uint32_t>(qr * kPartRowBytes + ((c ^ ((qr + owner) & 7)) << 4));
 }
 
+// 1/x and log2(x) by the PTX approximations (relative error about 2^-23, absolute error of the
+// logarithm about 2^-22 for normal x): one instruction each instead of the correctly rounded
+// sequences, whose dependent steps sit on the combine's chain with one warp per scheduler. The
+// output is rounded to bf16 (2^-9) and lse is held to 1e-3.
+__device__ __forceinline__ float rcp_approx(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float lg2_approx(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
   const __half2 h = __floats2half2_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&h);
@@ -404,7 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           am[c] = fmax3(am[c], fabsf(__uint_as_float(o[c][e])), fabsf(__uint_as_float(o[c][e + 1])));
       const float amax = fmaxf(fmaxf(am[0], am[1]), fmaxf(am[2], am[3]));
       const float sc = amax > 0.0f ? amax : 1.0f;
-      const float inv = 1.0f / sc;
+      const float inv = rcp_approx(sc);
       const int owner = R % nsplit, qr = R / nsplit;
       uint8_t* blk = stage + owner * rpo * kPartRowBytes;
 #pragma unroll
@@ -522,13 +537,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           acc.z = fmaf(pself, v23.x, acc.z);
           acc.w = fmaf(pself, v23.y, acc.w);
         }
-        const float inv = 1.0f / l;
+        const float inv = rcp_approx(l);
         const size_t orow = static_cast<size_t>(rowbase) + Pc;
         uint2 ov;
         ov.x = pack_bf16x2(acc.x * inv, acc.y * inv);
         ov.y = pack_bf16x2(acc.z * inv, acc.w * inv);
         reinterpret_cast<uint2*>(out + orow * kD)[lane] = ov;
-        if (lane == 0 && lse != nullptr) lse[orow] = (m + log2f(l)) * 0.6931471805599453f;
+        if (lane == 0 && lse != nullptr) lse[orow] = (m + lg2_approx(l)) * 0.6931471805599453f;
       }
     }
     // no CTA leaves while a copy out of its shared memory may still run (every owner has
