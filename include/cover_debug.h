@@ -69,11 +69,13 @@ int cover_debug_attn_fault(const void* q, const void* k_cached, const void* v_ca
  * limit_us > 0 it runs the kernel's self-test instance instead: CTA fault_cta
  * (grid order: key split fastest, then Q tile, KV head, batch row) leaves out
  * the K load of its first KV tile, and every bounded wait gives up after
- * limit_us microseconds (1 .. 2000000; 0: one second). That CTA records
- * COVER_ERR_DEVICE_TIMEOUT at site 60 or 61 (the first of its waits that
- * depend on the tile to give up), every role leaves its loop, and the
- * launch completes; the output rows of that CTA's cluster (its Q tile of its KV
- * head) are unspecified, every other row is the clean result. fault_cta = -1
+ * limit_us microseconds (1 .. 2000000; 0: one second). The first wait that
+ * depends on the missing tile to give up records COVER_ERR_DEVICE_TIMEOUT: at
+ * site 60 or 61 in that CTA, or at site 62 in a CTA of its cluster waiting for
+ * its partial block. Every role leaves its loop, every copy already issued
+ * lands before a CTA exits, and the launch completes. The output rows of that
+ * CTA's cluster (its Q tile of its KV head) are unspecified, and every other
+ * row is the clean result. fault_cta = -1
  * with limit_us = 0 is the normal launch. Arguments, layouts and errors as
  * cover_attn_fwd_prefix, plus COVER_ERR_INVALID_ARG for limit_us outside
  * 0 .. 2000000, and COVER_ERR_UNSUPPORTED where the packed kernel does not
@@ -85,6 +87,22 @@ int cover_debug_attn_prefix_packed(const void* q, const void* k_cached, const vo
                                    const int32_t* seed_idx, int n_seeds,
                                    int B, int Hq, int Hkv, int Lq, int Lk, int q0, int D,
                                    void* out, float* lse, int fault_cta, int limit_us, void* stream);
+
+/*
+ * The choice cover_attn_fwd_prefix makes for a bf16 window (Lq rows at memory
+ * positions q0.., an Lk-long memory, D = 128) between the packed grouped-query
+ * kernel and the square kernel, on a GPU with n_sm SMs where max_clusters[c-1]
+ * clusters of c CTAs of the packed kernel (c = 1 .. 8) can be resident at once
+ * (on the device the call queries both). Host arithmetic only: no device and
+ * no stream. Writes choice[6] = {supported, resident, packed, KV tiles per CTA,
+ * CTAs per cluster, Q tiles per KV head} (the last three 0 when unsupported)
+ * and times[2] = {predicted packed us, predicted square us} (0 when not
+ * computed). COVER_ERR_INVALID_ARG for B, Hq, Hkv < 1, Hq % Hkv != 0, an
+ * invalid window (as cover_attn_fwd_prefix), n_sm < 1, a negative count or a
+ * null pointer.
+ */
+int cover_debug_window_model(int B, int Hq, int Hkv, int Lq, int Lk, int q0, int n_sm,
+                             const int32_t* max_clusters, int32_t* choice, double* times);
 
 /*
  * Like cover_device_status, and also returns where the failure came from:

@@ -44,6 +44,7 @@ _SIGNATURES = {
     "cover_debug_attn_fault": (_I, [_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _P, _P, _I, _I, _I,
                                     _P]),
     "cover_debug_status_detail": (_I, [_P, _P]),
+    "cover_debug_window_model": (_I, [_I, _I, _I, _I, _I, _I, _I, _P, _P, _P]),
 }
 
 

@@ -460,6 +460,20 @@ def cover_debug_attn_fault(q, k_cached, v_cached, k_seedmask=None, v_seedmask=No
                         extra=(int(fault_cta), int(fault_entry), int(limit_us)))
 
 
+def cover_debug_window_model(B: int, Hq: int, Hkv: int, Lq: int, Lk: int, q0: int, n_sm: int, max_clusters):
+    """The prefix-window call's choice between the packed grouped-query kernel and the square kernel
+    on a GPU with n_sm SMs and max_clusters[c - 1] resident clusters of c packed CTAs (c = 1 .. 8).
+    Host arithmetic only (no device needed)."""
+    mc = (ctypes.c_int32 * 8)(*[int(x) for x in max_clusters])
+    choice = (ctypes.c_int32 * 6)()
+    times = (ctypes.c_double * 2)()
+    _lib.check("cover_debug_window_model",
+               _lib.load().cover_debug_window_model(B, Hq, Hkv, Lq, Lk, q0, n_sm, mc, choice, times))
+    return {"supported": bool(choice[0]), "resident": bool(choice[1]), "packed": bool(choice[2]),
+            "T": int(choice[3]), "nsplit": int(choice[4]), "n_qt": int(choice[5]),
+            "packed_us": float(times[0]), "square_us": float(times[1])}
+
+
 def cover_debug_status_detail(stream=None):
     """(status code, site id, block id) of the current device's status block, which is then cleared."""
     detail = (ctypes.c_int32 * 3)()

@@ -476,7 +476,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     // ---------------- combine ----------------
     // the nsplit blocks of this CTA's rows (copied by warp 4 of every CTA of the cluster)
-    if (!mbar_wait(&sm.bar_recv, 0, nullptr, wait_ns) && !sm.abort) {
+    const bool received = mbar_wait(&sm.bar_recv, 0, nullptr, wait_ns);
+    if (!received && !sm.abort) {
       report_status(status, kStatusTimeout, 62);
       sm.abort = 1;
     }
@@ -546,9 +547,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0 && lse != nullptr) lse[orow] = (m + lg2_approx(l)) * 0.6931471805599453f;
       }
     }
-    // no CTA leaves while a copy out of its shared memory may still run (every owner has
-    // received all of its blocks before it arrives)
+    // No CTA leaves while a copy out of its shared memory may still run: an owner arrives once
+    // it has received all of its blocks. An owner whose receive wait gave up (a sender of its
+    // cluster timed out before its copies) may not have them yet; but every CTA issues its
+    // copies before it arrives here, so after the barrier they are all in flight, and that owner
+    // waits for them to land before its shared memory is released.
     cluster_sync();
+    if (!received) mbar_wait(&sm.bar_recv, 0, nullptr, wait_ns);
   }
   if (warp == kMmaWarp) {
     cluster_wait();   // the prologue's arrival: every CTA of the cluster has its barriers set up
@@ -669,6 +674,27 @@ bool packed_supported(const AttnArgs& a) {
 
 }  // namespace
 
+WindowChoice window_gqa_model(const AttnArgs& a, int n_sm, const int* max_clusters) {
+  WindowChoice c{};
+  c.supported = packed_supported(a);
+  if (!c.supported) return c;
+  WinSetup su;
+  su.n_sm = n_sm;
+  su.max_clusters[0] = 0;
+  for (int cs = 1; cs <= kMaxSplit; ++cs) su.max_clusters[cs] = max_clusters[cs - 1];
+  const WinShape w = win_shape(a);
+  c.T = w.T;
+  c.nsplit = w.nsplit;
+  c.n_qt = w.n_qt;
+  c.clusters = w.clusters;
+  // a cluster of nsplit CTAs that cannot be resident leaves only the square kernel
+  c.resident = su.max_clusters[w.nsplit] >= 1;
+  c.packed_us = c.resident ? packed_us(w, su) : 0.0;
+  c.square_us = square_us(a, w, su);
+  c.packed = c.resident && c.packed_us < c.square_us;
+  return c;
+}
+
 int try_launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream, bool force) {
   const bool fault = a.fault_cta >= 0 || a.wait_ns > 0;
   // a self-test call of the square kernel never comes here unforced
@@ -677,9 +703,9 @@ int try_launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stre
   WinSetup su;
   const int rc = win_setup(&su, smem);
   if (rc != 0) return rc;
+  const WindowChoice ch = window_gqa_model(a, su.n_sm, su.max_clusters + 1);
+  if (!ch.resident || (!force && !ch.packed)) return kWindowGqaNotTaken;
   const WinShape w = win_shape(a);
-  if (su.max_clusters[w.nsplit] < 1) return kWindowGqaNotTaken;   // such a cluster cannot be resident
-  if (!force && packed_us(w, su) >= square_us(a, w, su)) return kWindowGqaNotTaken;
   const long long grid = w.clusters * w.nsplit;
   if (grid > 0x7fffffffLL) return -2;
   CUtensorMap tq, tk, tv;

@@ -369,6 +369,29 @@ int cover_debug_attn_prefix_packed(const void* q, const void* k_cached, const vo
   return rc == cover::kWindowGqaNotTaken ? COVER_ERR_UNSUPPORTED : rc;
 }
 
+int cover_debug_window_model(int B, int Hq, int Hkv, int Lq, int Lk, int q0, int n_sm, const int32_t* max_clusters,
+                             int32_t* choice, double* times) {
+  if (B < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || n_sm < 1 || max_clusters == nullptr || choice == nullptr ||
+      times == nullptr)
+    return COVER_ERR_INVALID_ARG;
+  const int rc = check_window(Lq, Lk, q0);
+  if (rc != COVER_OK) return rc;
+  for (int c = 0; c < 8; ++c)
+    if (max_clusters[c] < 0) return COVER_ERR_INVALID_ARG;
+  cover::AttnArgs a{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, 0, B, Hq, Hkv, Lk, 128, nullptr, nullptr,
+                    Lq, q0};
+  const cover::WindowChoice c = cover::window_gqa_model(a, n_sm, max_clusters);
+  choice[0] = c.supported;
+  choice[1] = c.resident;
+  choice[2] = c.packed;
+  choice[3] = c.T;
+  choice[4] = c.nsplit;
+  choice[5] = c.n_qt;
+  times[0] = c.packed_us;
+  times[1] = c.square_us;
+  return COVER_OK;
+}
+
 int cover_debug_attn_fault(const void* q, const void* k_cached, const void* v_cached, const void* k_seedmask,
                            const void* v_seedmask, const int32_t* seed_idx, int n_seeds, int B, int Hq, int Hkv,
                            int Lq, int Lk, int q0, int D, void* out, float* lse, int fault_cta, int fault_entry,

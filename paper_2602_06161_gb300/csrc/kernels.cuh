@@ -43,6 +43,17 @@ constexpr int kMaxWindowGqaPacked = 1024;
 constexpr int kMaxWindowGqaSteps = 8;
 constexpr int kWindowGqaNotTaken = 1;
 int try_launch_attn_window_gqa(const AttnArgs& a, int* status, cudaStream_t stream, bool force);
+// The launch-time choice for a window on a GPU with n_sm SMs, where max_clusters[c - 1] clusters
+// of c CTAs of the packed kernel can be resident at once (c = 1 .. 8). Host arithmetic only.
+struct WindowChoice {
+  bool supported;          // the packed kernel runs this shape
+  bool resident;           // a cluster of its nsplit CTAs can be resident
+  bool packed;             // it is predicted faster than the square kernel
+  int T, nsplit, n_qt;     // KV tiles per CTA, CTAs per cluster, Q tiles per KV head
+  long long clusters;
+  double packed_us, square_us;
+};
+WindowChoice window_gqa_model(const AttnArgs& a, int n_sm, const int* max_clusters);
 int launch_attn_f32(const AttnArgs& a, int* status, cudaStream_t stream);
 
 int launch_seed_route(const int32_t* seed_idx, int n_seeds, int B, int L, int32_t* slot_out, uint32_t* bitmap_out,
